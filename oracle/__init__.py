@@ -1,0 +1,236 @@
+"""Float64 CPU oracle for the Scale-QLoRA scale-only training step (numpy front end).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the
+benchmark's ``cpu_baseline`` / ``--impl reference`` legs may import this module;
+the product path (``paper_2609_04526_gb300``) never does. The arithmetic lives in
+``sq_oracle.c`` (plain loops, float64 accumulation), which shares no code with the
+CUDA sources. Each wrapper names the paper passage its C function follows.
+"""
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+NVFP4 = 0
+MXFP4 = 1
+BLOCK = {NVFP4: 16, MXFP4: 32}
+
+_lib = None
+
+_i64 = ctypes.c_int64
+_p = ctypes.c_void_p
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        path = _build.build()
+        L = ctypes.CDLL(path)
+        L.or_e2m1.restype = ctypes.c_double
+        L.or_e2m1.argtypes = [ctypes.c_int]
+        L.or_e4m3.restype = ctypes.c_double
+        L.or_e4m3.argtypes = [ctypes.c_int]
+        L.or_e8m0.restype = ctypes.c_double
+        L.or_e8m0.argtypes = [ctypes.c_int]
+        L.or_e4m3_rne.restype = ctypes.c_int
+        L.or_e4m3_rne.argtypes = [ctypes.c_float]
+        L.or_round_log2.restype = ctypes.c_int
+        L.or_round_log2.argtypes = [ctypes.c_float]
+        L.or_decode_weight.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _p]
+        L.or_fwd_f64.argtypes = [_i64, _i64, _i64, _p, _p, _p]
+        L.or_dx_f64.argtypes = [_i64, _i64, _i64, _p, _p, _p]
+        L.or_scale_grad_f64.argtypes = [_i64, _i64, _i64, ctypes.c_int, _p, _p, _p, _p, _i64, _p, _p]
+        L.or_fwd.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _p]
+        L.or_dx.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _p]
+        L.or_scale_grad.argtypes = [ctypes.c_int, _i64, _i64, _p, _i64, _p, _p, _p, _i64, _p, _p]
+        L.or_fwd_at.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _i64, _p, _p, _p]
+        L.or_dx_at.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _i64, _p, _p, _p]
+        L.or_project.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
+        L.or_merge.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
+        L.or_num_threads.restype = ctypes.c_int
+        _lib = L
+    return _lib
+
+
+def _ptr(a):
+    return a.ctypes.data_as(ctypes.c_void_p) if a is not None else None
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def num_threads() -> int:
+    return int(lib().or_num_threads())
+
+
+# --- format decode (Sec. 2) -------------------------------------------------
+
+def e2m1(nibble: int) -> float:
+    return lib().or_e2m1(int(nibble))
+
+
+def e4m3(byte: int) -> float:
+    return lib().or_e4m3(int(byte))
+
+
+def e8m0(byte: int) -> float:
+    return lib().or_e8m0(int(byte))
+
+
+def e4m3_rne(q: float) -> int:
+    return lib().or_e4m3_rne(float(q))
+
+
+def round_log2(L: float) -> int:
+    return lib().or_round_log2(float(L))
+
+
+def decode_weight(fmt, codes, scales, ws2, N, K):
+    """W[n,k] = code[n,k] * eff_scale[n, k // block] in float64 (Sec. 2)."""
+    codes = _c(codes, np.uint8)
+    scales = _c(scales, np.uint8)
+    W = np.empty((N, K), dtype=np.float64)
+    lib().or_decode_weight(fmt, N, K, _ptr(codes), _ptr(scales), float(ws2), _ptr(W))
+    return W
+
+
+# --- contractions on float64 operands ---------------------------------------
+
+def fwd_f64(X, W):
+    """Y = X W^T (Sec. 3 forward)."""
+    X = _c(X, np.float64)
+    W = _c(W, np.float64)
+    M, K = X.shape
+    N = W.shape[0]
+    Y = np.empty((M, N), dtype=np.float64)
+    lib().or_fwd_f64(M, N, K, _ptr(X), _ptr(W), _ptr(Y))
+    return Y
+
+
+def dx_f64(dY, W):
+    """dX = dY W (input gradient of Y = X W^T)."""
+    dY = _c(dY, np.float64)
+    W = _c(W, np.float64)
+    M, N = dY.shape
+    K = W.shape[1]
+    dX = np.empty((M, K), dtype=np.float64)
+    lib().or_dx_f64(M, N, K, _ptr(dY), _ptr(W), _ptr(dX))
+    return dX
+
+
+def scale_grad_f64(fmt, codes, X, dY, mask=None, rows=None):
+    """g[n,b] = sum_{k in b} code[n,k] (dY^T X)[n,k], optionally times mask[n,b]."""
+    X = _c(X, np.float64)
+    dY = _c(dY, np.float64)
+    codes = _c(codes, np.uint8)
+    M, K = X.shape
+    N = dY.shape[1]
+    B = BLOCK[fmt]
+    G = K // B
+    mask_a = _c(mask, np.uint8) if mask is not None else None
+    if rows is None:
+        g = np.empty((N, G), dtype=np.float64)
+        lib().or_scale_grad_f64(M, N, K, B, _ptr(codes), _ptr(X), _ptr(dY), _ptr(mask_a), 0, None, _ptr(g))
+    else:
+        rows = _c(rows, np.int64)
+        g = np.empty((len(rows), G), dtype=np.float64)
+        lib().or_scale_grad_f64(M, N, K, B, _ptr(codes), _ptr(X), _ptr(dY), _ptr(mask_a), len(rows),
+                                _ptr(rows), _ptr(g))
+    return g
+
+
+# --- entry points on packed formats (bf16 activations as uint16 bit patterns) --
+
+def fwd(fmt, codes, scales, ws2, X_bits):
+    X_bits = _c(X_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    scales = _c(scales, np.uint8)
+    M, K = X_bits.shape
+    N = codes.shape[0]
+    Y = np.empty((M, N), dtype=np.float64)
+    lib().or_fwd(fmt, N, K, _ptr(codes), _ptr(scales), float(ws2), M, _ptr(X_bits), _ptr(Y))
+    return Y
+
+
+def dx(fmt, codes, scales, ws2, dY_bits):
+    dY_bits = _c(dY_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    scales = _c(scales, np.uint8)
+    M, N = dY_bits.shape
+    K = codes.shape[1] * 2
+    dX = np.empty((M, K), dtype=np.float64)
+    lib().or_dx(fmt, N, K, _ptr(codes), _ptr(scales), float(ws2), M, _ptr(dY_bits), _ptr(dX))
+    return dX
+
+
+def scale_grad(fmt, codes, X_bits, dY_bits, mask=None, rows=None):
+    X_bits = _c(X_bits, np.uint16)
+    dY_bits = _c(dY_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    M, K = X_bits.shape
+    N = dY_bits.shape[1]
+    G = K // BLOCK[fmt]
+    mask_a = _c(mask, np.uint8) if mask is not None else None
+    if rows is None:
+        g = np.empty((N, G), dtype=np.float64)
+        lib().or_scale_grad(fmt, N, K, _ptr(codes), M, _ptr(X_bits), _ptr(dY_bits), _ptr(mask_a), 0, None,
+                            _ptr(g))
+    else:
+        rows = _c(rows, np.int64)
+        g = np.empty((len(rows), G), dtype=np.float64)
+        lib().or_scale_grad(fmt, N, K, _ptr(codes), M, _ptr(X_bits), _ptr(dY_bits), _ptr(mask_a), len(rows),
+                            _ptr(rows), _ptr(g))
+    return g
+
+
+def fwd_at(fmt, codes, scales, ws2, X_bits, ms, ns):
+    X_bits = _c(X_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    scales = _c(scales, np.uint8)
+    ms = _c(ms, np.int64)
+    ns = _c(ns, np.int64)
+    M, K = X_bits.shape
+    N = codes.shape[0]
+    out = np.empty(len(ms), dtype=np.float64)
+    lib().or_fwd_at(fmt, N, K, _ptr(codes), _ptr(scales), float(ws2), M, _ptr(X_bits), len(ms), _ptr(ms),
+                    _ptr(ns), _ptr(out))
+    return out
+
+
+def dx_at(fmt, codes, scales, ws2, dY_bits, ms, ks):
+    dY_bits = _c(dY_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    scales = _c(scales, np.uint8)
+    ms = _c(ms, np.int64)
+    ks = _c(ks, np.int64)
+    M, N = dY_bits.shape
+    K = codes.shape[1] * 2
+    out = np.empty(len(ms), dtype=np.float64)
+    lib().or_dx_at(fmt, N, K, _ptr(codes), _ptr(scales), float(ws2), M, _ptr(dY_bits), len(ms), _ptr(ms),
+                   _ptr(ks), _ptr(out))
+    return out
+
+
+# --- projection and merge (Sec. 3 QAST round_grid, clamp; Sec. 5 rollback) ---
+
+def project(fmt, latent, ws2):
+    """Returns (bytes, mask, nonfinite) for a latent scale plane (any shape)."""
+    L = _c(latent, np.float32)
+    out = np.empty(L.shape, dtype=np.uint8)
+    mask = np.empty(L.shape, dtype=np.uint8)
+    nf = ctypes.c_int64(0)
+    lib().or_project(fmt, L.size, float(ws2), _ptr(L), _ptr(out), _ptr(mask), ctypes.byref(nf))
+    return out, mask, int(nf.value)
+
+
+def merge(fmt, latent, scales, ws2, want_delta=True):
+    """Returns (new_scales, delta or None, changed). `scales` is not modified."""
+    L = _c(latent, np.float32)
+    s = np.array(scales, dtype=np.uint8, copy=True, order="C")
+    delta = np.empty(L.shape, dtype=np.float32) if want_delta else None
+    ch = ctypes.c_int64(0)
+    lib().or_merge(fmt, L.size, float(ws2), _ptr(L), _ptr(s), _ptr(delta), ctypes.byref(ch))
+    return s, delta, int(ch.value)
