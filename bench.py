@@ -1,0 +1,462 @@
+#!/usr/bin/env python
+"""Benchmark of the Scale-QLoRA scale-only training step on a Llama-3-8B-shaped
+NVFP4 decoder layer (q, k, v, o, gate, up, down; 16 x 2048 tokens).
+
+One step = for every linear: grid projection of the latent scales (with STE
+mask), forward, input gradient, masked block-reduced scale gradient, and the
+merge of the latent into the artifact's scale plane: every row of the hot path.
+Metric: fwd+dX+dScale TFLOP/s = 6*M*N*K summed over the linears / step time,
+with its fraction of the measured GB300 dense-bf16 peak.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (launched by torch.distributed.run) every rank runs an independent
+replica of the step (the method has no exchange on this path); rank 0 prints
+the JSON line with the maximum time over ranks. `--impl reference` times the
+float64 CPU oracle on a bounded sample of the same workload on the host cores.
+"""
+import argparse
+import json
+import os
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "fwd+dX+dScale TFLOP/s per layer & fraction of GB300 bf16 tensor peak"
+UNIT = "TFLOP/s"
+KINDS = ("project", "fwd", "dx", "sgrad", "merge")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default="c5")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16": float(p["bf16_tflops"]),
+                "bf16_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+# --------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of SM clock and throttle reasons during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.path = None
+        exe = shutil.which("nvidia-smi")
+        if not exe:
+            return
+        try:
+            uuid = "GPU-" + str(torch.cuda.get_device_properties(device_index).uuid)
+        except Exception:
+            uuid = None
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        cmd = [exe] + (["-i", uuid] if uuid else []) + ["--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                                                         "-lms", "200"]
+        self.fh = open(self.path, "w")
+        self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 8:
+                    continue
+                try:
+                    sm.append(float(parts[0]))
+                    smax.append(float(parts[1]))
+                except ValueError:
+                    continue
+                for name, v in zip(names, parts[4:8]):
+                    if v.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------- workload
+
+class LayerState:
+    """Device-resident inputs and outputs of one step of the workload."""
+
+    def __init__(self, wl, device):
+        import paper_2609_04526_gb300 as pkg
+        from paper_2609_04526_gb300 import synth
+        self.wl = wl
+        self.lin = []
+        self.acts = {name: synth.gen_act(wl, name, device=device) for name in synth.act_names(wl)}
+        for lin in wl.linears:
+            w = synth.gen_weight(wl, lin, device=device)
+            L = synth.gen_latent(wl, lin, w, device=device)
+            G = lin.K // wl.block
+            st = dict(
+                lin=lin, base_scales=w.scales, ws2=w.ws2, codes=w.codes, latent=L,
+                art=w.scales.clone(),                       # artifact scale plane rewritten by the merge
+                qbytes=torch.empty_like(w.scales),          # projected (on-grid) scale bytes used by the forward
+                mask=torch.empty_like(w.scales),
+                dY=synth.gen_dy(wl, lin, device=device),
+                Y=torch.empty(wl.M, lin.N, dtype=torch.bfloat16, device=device),
+                dX=torch.empty(wl.M, lin.K, dtype=torch.bfloat16, device=device),
+                g=torch.empty(lin.N, G, dtype=torch.float32, device=device),
+                nonfinite=torch.zeros(1, dtype=torch.int32, device=device),
+                changed=torch.zeros(1, dtype=torch.int64, device=device),
+            )
+            st["qw"] = pkg.QuantWeight(wl.fmt, lin.N, lin.K, w.codes, st["qbytes"], w.ws2)
+            self.lin.append(st)
+
+    def inputs(self):
+        """(name, tensor) of every per-step input: activations, output gradients, latent scales."""
+        out = [("X:" + k, v) for k, v in self.acts.items()]
+        for st in self.lin:
+            out.append(("dY:" + st["lin"].name, st["dY"]))
+            out.append(("L:" + st["lin"].name, st["latent"]))
+        return out
+
+    def results(self):
+        """(name, tensor) of the step's results read back by a user: scale gradients,
+        merged scale planes and the NaN / changed-byte counters."""
+        out = []
+        for st in self.lin:
+            out += [("g:" + st["lin"].name, st["g"]), ("art:" + st["lin"].name, st["art"]),
+                    ("nf:" + st["lin"].name, st["nonfinite"]), ("ch:" + st["lin"].name, st["changed"])]
+        return out
+
+
+def run_step(h, S, stream, events=None):
+    fmt = S.wl.fmt
+    for i, st in enumerate(S.lin):
+        X = S.acts[st["lin"].x]
+        ev = events[i] if events is not None else None
+        if ev:
+            ev[0].record(stream)
+        h.sq_project_scales(fmt, st["latent"], st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
+                            nonfinite=st["nonfinite"], stream=stream)
+        if ev:
+            ev[1].record(stream)
+        h.sq_fwd(st["qw"], X, st["Y"], stream=stream)
+        if ev:
+            ev[2].record(stream)
+        h.sq_bwd_dx(st["qw"], st["dY"], st["dX"], stream=stream)
+        if ev:
+            ev[3].record(stream)
+        h.sq_scale_grad(st["qw"], X, st["dY"], mask=st["mask"], g=st["g"], stream=stream)
+        if ev:
+            ev[4].record(stream)
+        h.sq_merge(fmt, st["latent"], st["ws2"], st["art"], changed=st["changed"], stream=stream)
+        if ev:
+            ev[5].record(stream)
+
+
+LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge kernels
+
+
+def kernel_work(S):
+    """Algorithmic FLOPs (contractions) and bytes (projection / merge) per kernel kind per step."""
+    fl = {"fwd": 0, "dx": 0, "sgrad": 0}
+    by = {"project": 0, "merge": 0}
+    for st in S.lin:
+        l = st["lin"]
+        for k in fl:
+            fl[k] += 2 * S.wl.M * l.N * l.K
+        blocks = l.N * (l.K // S.wl.block)
+        by["project"] += blocks * (4 + 1 + 1)   # latent fp32 in, byte + mask byte out
+        by["merge"] += blocks * (4 + 1 + 1)     # latent in, old byte in, new byte out
+    return fl, by
+
+
+# --------------------------------------------------------------------- oracle sample
+
+def oracle_sample(wl, host, linears, n_y, n_dx, n_rows, n_plane, seed=0):
+    """Time the float64 oracle on a bounded sample of one step and extrapolate
+    the full step's CPU time from each part's per-unit rate."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    t_full = 0.0
+    t_spent = 0.0
+    desc = []
+    for lin in linears:
+        d = host[lin.name]
+        M, N, K = wl.M, lin.N, lin.K
+        ms, ns, ks = rng.integers(0, M, n_y), rng.integers(0, N, n_y), rng.integers(0, K, n_dx)
+        t0 = time.perf_counter()
+        oracle.fwd_at(wl.fmt, d["codes"], d["scales"], d["ws2"], d["X"], ms, ns)
+        t1 = time.perf_counter()
+        oracle.dx_at(wl.fmt, d["codes"], d["scales"], d["ws2"], d["dY"], ms[:n_dx], ks)
+        t2 = time.perf_counter()
+        rows = rng.integers(0, N, n_rows)
+        oracle.scale_grad(wl.fmt, d["codes"], d["X"], d["dY"], mask=d["mask"], rows=rows)
+        t3 = time.perf_counter()
+        Lp = d["latent"].reshape(-1)[:n_plane]
+        oracle.project(wl.fmt, Lp, d["ws2"])
+        t4 = time.perf_counter()
+        oracle.merge(wl.fmt, Lp, d["scales"].reshape(-1)[:n_plane], d["ws2"], want_delta=False)
+        t5 = time.perf_counter()
+        blocks = N * (K // wl.block)
+        t_full += ((t1 - t0) * (M * N / n_y) + (t2 - t1) * (M * K / n_dx) + (t3 - t2) * (N / n_rows)
+                   + (t4 - t3 + t5 - t4) * (blocks / min(n_plane, blocks)))
+        t_spent += t5 - t0
+        desc.append(lin.name)
+    return t_full, t_spent, (f"{n_y} Y and {n_dx} dX elements, {n_rows} full scale-gradient rows and "
+                             f"{n_plane} latents through projection and merge, per linear ({', '.join(desc)}); "
+                             "full-step time extrapolated from each part's measured per-element rate")
+
+
+def host_copies(S, linears):
+    out = {}
+    for st in S.lin:
+        l = st["lin"]
+        if l not in linears:
+            continue
+        X = S.acts[l.x]
+        out[l.name] = dict(
+            codes=st["codes"].cpu().numpy(), scales=st["base_scales"].cpu().numpy(), ws2=st["ws2"],
+            X=X.cpu().contiguous().view(torch.int16).numpy().view(np.uint16),
+            dY=st["dY"].cpu().contiguous().view(torch.int16).numpy().view(np.uint16),
+            mask=st["mask"].cpu().numpy(), latent=st["latent"].cpu().numpy())
+    return out
+
+
+# --------------------------------------------------------------------- arms
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and not torch.distributed.is_initialized():
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        torch.distributed.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def run_ours(args):
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import build, synth
+    world, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    build.build()
+    wl = synth.WORKLOADS[args.workload]
+    pk = peaks()
+    S = LayerState(wl, "cuda")
+    h = pkg.Handle()
+    stream = torch.cuda.current_stream()
+    flops_step = wl.flops()
+
+    for _ in range(args.warmup):
+        run_step(h, S, stream)
+    h.sq_sync(stream)
+
+    # ---- device-resident timed region (inputs already in HBM; inputs > L2)
+    nl = len(S.lin)
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(nl)] for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    t_start.record(stream)
+    for k in range(args.steps):
+        run_step(h, S, stream, events[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    h.sq_sync(stream)
+    ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
+    ms_step = ms_total / args.steps
+
+    kind_ms = {k: 0.0 for k in KINDS}
+    kind_launch = {k: 0 for k in KINDS}
+    for k in range(args.steps):
+        for i in range(nl):
+            ev = events[k][i]
+            for j, kind in enumerate(KINDS):
+                kind_ms[kind] += ev[j].elapsed_time(ev[j + 1])
+                kind_launch[kind] += 1
+    fl, by = kernel_work(S)
+    kernels = {}
+    for kind in KINDS:
+        t = kind_ms[kind] / args.steps / 1e3  # s per step
+        if kind in fl:
+            ach = fl[kind] / t / 1e12
+            kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "TFLOP/s",
+                             "frac": ach / pk["bf16_sustained"]}
+        else:
+            ach = by[kind] / t / 1e9
+            kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
+    dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
+    value = flops_step * args.steps * world / (ms_total / 1e3) / 1e12
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        ins = [(n, t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for n, t in S.inputs()]
+        outs = [(n, t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for n, t in S.results()]
+        for _, dev, hst in ins:
+            hst.copy_(dev)
+        h2d = sum(t.numel() * t.element_size() for _, t, _ in ins)
+        d2h = sum(t.numel() * t.element_size() for _, t, _ in outs)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            for _, dev, hst in ins:
+                dev.copy_(hst, non_blocking=True)
+            run_step(h, S, stream)
+            for _, dev, hst in outs:
+                hst.copy_(dev, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        h.sq_sync(stream)
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+        e2e = {"value": flops_step * args.steps * world / (e2e_ms / 1e3) / 1e12, "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps}
+
+    # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.lib()
+        host = host_copies(S, list(wl.linears))
+        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=256, n_dx=256, n_rows=4,
+                                              n_plane=1 << 17)
+        cpu = {"value": flops_step / t_full / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+               "sample": desc, "sample_seconds": round(t_spent, 2), "extrapolated_step_seconds": round(t_full, 1)}
+
+    if rank == 0:
+        k = kernels[dom]
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": f"{wl.key}: {wl.title}", "M": wl.M,
+                       "linears": {l.name: [l.N, l.K] for l in wl.linears}, "format": "nvfp4" if wl.fmt == 0 else "mxfp4",
+                       "l2": "inputs larger than L2 (activations + output gradients > 4 GB per step), no flush",
+                       "parallelism": f"replicas x{world}", "flops_per_step": flops_step},
+            "roofline": {"bound": "tensor", "kernel": dom, "achieved": k["achieved"],
+                         "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": k["achieved"] / pk["bf16_sustained"],
+                         "traffic": None, "peak_source": f"{pk['source']} bf16 sustained"},
+            "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
+            "kernels": kernels,
+            "e2e": e2e, "cpu_baseline": cpu,
+            "gpu_launches": LAUNCHES_PER_LINEAR * nl * args.steps,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def run_reference(args):
+    """The float64 CPU oracle, as it stands, on bounded samples of the same workload."""
+    world, rank, local = dist_setup(args)
+    if rank != 0:
+        return
+    import oracle
+    from paper_2609_04526_gb300 import synth
+    oracle.lib()
+    wl = synth.WORKLOADS[args.workload]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    if dev == "cuda":
+        torch.cuda.set_device(local)
+    host = {}
+    acts = {}
+    for lin in wl.linears:
+        w = synth.gen_weight(wl, lin, device=dev)
+        if lin.x not in acts:
+            acts[lin.x] = synth.gen_act(wl, lin.x, device=dev).cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        L = synth.gen_latent(wl, lin, w, device=dev)
+        G = lin.K // wl.block
+        host[lin.name] = dict(codes=w.codes.cpu().numpy(), scales=w.scales.cpu().numpy(), ws2=w.ws2, X=acts[lin.x],
+                              dY=synth.gen_dy(wl, lin, device=dev).cpu().contiguous().view(torch.int16).numpy().view(np.uint16),
+                              mask=np.ones((lin.N, G), dtype=np.uint8), latent=L.cpu().numpy())
+        del w, L
+    lins = list(wl.linears)
+    per_step = []
+    for k in range(args.warmup + args.steps):
+        lin = lins[k % len(lins)]
+        t_full, t_spent, desc = oracle_sample(wl, host, [lin], n_y=64, n_dx=64, n_rows=1, n_plane=1 << 15, seed=k)
+        # scale this linear's extrapolated time to the whole layer by its FLOP share
+        share = 6 * wl.M * lin.N * lin.K / wl.flops()
+        if k >= args.warmup:
+            per_step.append((t_full / share, t_spent))
+    t_layer = statistics.median(t for t, _ in per_step)
+    value = wl.flops() / t_layer / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(s for _, s in per_step), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{wl.key}: {wl.title}", "M": wl.M, "format": "nvfp4" if wl.fmt == 0 else "mxfp4",
+                   "parallelism": "host cores"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": "each step: one linear (cycling through the 7), 64 Y and 64 dX elements, one full "
+                                   "scale-gradient row, 32768 latents through projection and merge; full-layer time "
+                                   "extrapolated from per-element rates and the linear's FLOP share (median over steps)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+    if torch.distributed.is_available() and torch.distributed.is_initialized():
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,139 @@
+/*
+ * scaleqlora.h -- C ABI of the GB300 (sm_103a) hot path of Scale-QLoRA's
+ * scale-only training step (arXiv 2609.04526).
+ *
+ * The E2M1 code plane of a native FP4 checkpoint is frozen; only the per-block
+ * scales train. Per linear layer with weight W[N=out, K=in]:
+ *   sq_fwd             Y  = X . W^T                        (Sec. 3 "Scale-QLoRA forward")
+ *   sq_bwd_dx          dX = dY . W                         (backward of that forward)
+ *   sq_scale_grad      g[n,b] = sum_{k in b} code[n,k] (dY^T X)[n,k]   (optionally x mask)
+ *   sq_project_scales  latent scale -> on-grid E4M3 / E8M0 byte + STE mask (Sec. 3 QAST, clamp)
+ *   sq_merge           write on-grid bytes into the scale plane; never a code (Sec. 3, Sec. 5)
+ * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
+ *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
+ *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
+ *
+ * Conventions for every entry point
+ *  - Pointers named as device buffers are device pointers owned by the caller;
+ *    the library never frees or keeps them. Calls are asynchronous on `stream`
+ *    (a cudaStream_t passed as void*, NULL = the legacy default stream) and
+ *    return once the work is enqueued.
+ *  - Layouts are dense row-major. bf16 tensors are passed as uint16_t bit patterns.
+ *  - codes [N, K/2] u8: element k of row n is nibble (k & 1) of byte k/2, the even
+ *    k in the low nibble. scales [N, K/B] u8.
+ *  - Shape rules: N > 0 with N % 8 == 0; K > 0 with K % 32 == 0; M >= 0 (M == 0
+ *    is an empty batch). Every device pointer must be 16-byte aligned.
+ *  - Argument errors return SQ_ERR_INVALID_ARG before anything is launched; the
+ *    text is in sq_last_error(h). No exception or abort crosses the ABI.
+ *  - A handle is not thread-safe; use one handle per host thread.
+ *  - Device waits are bounded: a wait that runs out sets a device error word
+ *    instead of hanging; sq_sync reports it as SQ_ERR_DEVICE_TIMEOUT.
+ *  - Decoded weights are formed exactly in bf16 (the code x scale-byte product
+ *    has at most 6 significant bits); for MXFP4 this holds for scale bytes 2..252
+ *    (decoded magnitudes within bf16's normal range).
+ */
+#ifndef SCALEQLORA_H
+#define SCALEQLORA_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SQ_NVFP4 = 0, /* block 16, E4M3 scale byte times an fp32 tensor scale ws2 */
+  SQ_MXFP4 = 1  /* block 32, E8M0 power-of-two scale byte */
+} sq_format;
+
+typedef enum {
+  SQ_OK = 0,
+  SQ_ERR_INVALID_ARG = -1,    /* bad pointer, alignment, shape or scalar          */
+  SQ_ERR_UNSUPPORTED = -2,    /* current device is not compute capability 10.3    */
+  SQ_ERR_DEVICE = -3,         /* no usable CUDA device / driver entry point        */
+  SQ_ERR_CUDA = -4,           /* a CUDA runtime call or launch failed             */
+  SQ_ERR_DEVICE_TIMEOUT = -5  /* a bounded device-side wait ran out (see sq_sync)  */
+} sq_status;
+
+/* Opaque per-thread context: last error text, device properties, the device
+ * error word. */
+typedef struct sq_handle_s *sq_handle;
+
+/* One quantized linear, weight [N = out features, K = in features]. */
+typedef struct {
+  int32_t fmt;           /* sq_format                                           */
+  int32_t N;             /* out features, N % 8 == 0                            */
+  int32_t K;             /* in features,  K % 32 == 0                           */
+  const uint8_t *codes;  /* device [N, K/2]: packed E2M1 codes                  */
+  const uint8_t *scales; /* device [N, K/B]: E4M3 (NVFP4) or E8M0 (MXFP4) bytes */
+  float ws2;             /* NVFP4: finite and > 0; MXFP4: exactly 1.0           */
+} sq_weight;
+
+/* Create / destroy a handle. sq_create makes no CUDA call; the device is
+ * queried on the first compute call. */
+sq_status sq_create(sq_handle *out);
+sq_status sq_destroy(sq_handle h);
+
+/* Static text for a status code; never NULL. */
+const char *sq_status_string(sq_status s);
+/* Text of the last error on this handle ("" if none). Valid until the next call. */
+const char *sq_last_error(sq_handle h);
+
+/* Synchronise `stream` and report device-side wait timeouts raised since the
+ * previous sq_sync on this handle's device (then clear them).
+ * Returns SQ_OK, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
+sq_status sq_sync(sq_handle h, void *stream);
+
+/* Forward, Sec. 3 "Scale-QLoRA forward": Y[m,n] = sum_k X[m,k] W[n,k].
+ * X  device bf16 [M, K] (input), Y device bf16 [M, N] (output, overwritten).
+ * Accumulation in fp32; ws2 is applied to the fp32 accumulator; Y is rounded
+ * to nearest-even bf16. */
+sq_status sq_fwd(sq_handle h, const sq_weight *w, const uint16_t *X, int64_t M, uint16_t *Y, void *stream);
+
+/* Input gradient of the forward: dX[m,k] = sum_n dY[m,n] W[n,k].
+ * dY device bf16 [M, N] (input), dX device bf16 [M, K] (output). fp32 accumulation. */
+sq_status sq_bwd_dx(sq_handle h, const sq_weight *w, const uint16_t *dY, int64_t M, uint16_t *dX, void *stream);
+
+/* Scale gradient with respect to the effective scale s[n,b] (absolute units):
+ *   g[n,b] = mask[n,b] * sum_{k in block b} code[n,k] * sum_m dY[m,n] X[m,k]
+ * The derivative of sum(Y * dY) by s[n,b] under the forward above (Sec. 3), with
+ * the QAST straight-through estimator passing it unchanged through the grid
+ * rounding and the clamp zeroing it where the latent is outside the clamp
+ * (mask from sq_project_scales; NULL means all ones). The gradient of the
+ * latent in E4M3 units is g * ws2 (not computed here).
+ * X device bf16 [M, K], dY device bf16 [M, N], mask device u8 [N, K/B] or NULL,
+ * g device fp32 [N, K/B] (output, overwritten; all zero when M == 0). The
+ * weight's scale bytes are not read (w->scales may be NULL).
+ * The dW = dY^T X tile is reduced per block on chip and never written. */
+sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
+                        const uint8_t *mask, float *g, void *stream);
+
+/* Grid projection, Sec. 3 QAST round_grid with the ceiling clamp of the
+ * stability recipe (ii)/(iii), for count = N*G latent scales (absolute units):
+ *  NVFP4: cap = fl32(448*ws2); q = fl32(clamp(L, -cap, cap) / ws2);
+ *         byte = E4M3 nearest to q, ties to even (sign kept, -0 -> 0x80);
+ *         mask = 1 iff -cap <= L <= cap; NaN -> 0x7F with mask 0.
+ *  MXFP4: byte = round(log2 L) + 127 with the rounding at sqrt(2) * 2^E, clamped
+ *         to [0, 254] (mask 0 when clamped); L <= 0 -> 0 with mask 0;
+ *         +inf -> 254 with mask 0; NaN -> 0xFF with mask 0.
+ * latent device fp32 [N, G]; bytes_out device u8 [N, G]; mask_out device u8
+ * [N, G] or NULL; nonfinite device int32 or NULL: set to the number of NaN
+ * latents (written on `stream`). */
+sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
+                            uint8_t *bytes_out, uint8_t *mask_out, int32_t *nonfinite, void *stream);
+
+/* Merge, Sec. 3 "QAST makes merge exact by construction": rewrite the artifact's
+ * scale plane in place with the projection above (the same clamp and grid
+ * path) of `latent`. No code pointer is taken, so no code byte can change.
+ * scales_inout device u8 [N, G]; ongrid_delta device fp32 [N, G] or NULL:
+ *   fl32(s(new) - s(old)) with s(byte) = fl32(E4M3(byte) * ws2) or E8M0(byte),
+ *   the delta whose subtraction restores the base (Sec. 5, Payoff 3);
+ * changed_bytes device int64 or NULL: set to the number of bytes that changed. */
+sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
+                   uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SCALEQLORA_H */

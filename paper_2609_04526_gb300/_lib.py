@@ -1,0 +1,182 @@
+"""ctypes binding of libscaleqlora (include/scaleqlora.h).
+
+Argument marshalling only: torch tensors supply device pointers and the current
+CUDA stream; every step of the path runs in the library's kernels. There is no
+fallback: if the shared library is missing, loading raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libscaleqlora.so")
+
+NVFP4 = 0
+MXFP4 = 1
+BLOCK = {NVFP4: 16, MXFP4: 32}
+
+SQ_OK = 0
+STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "SQ_ERR_DEVICE", -4: "SQ_ERR_CUDA",
+          -5: "SQ_ERR_DEVICE_TIMEOUT"}
+
+# Every entry point the header declares (checked against include/scaleqlora.h by the tests).
+EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
+           "sq_scale_grad", "sq_project_scales", "sq_merge")
+
+
+class SQError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class _SqWeight(ctypes.Structure):
+    _fields_ = [("fmt", ctypes.c_int32), ("N", ctypes.c_int32), ("K", ctypes.c_int32),
+                ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("ws2", ctypes.c_float)]
+
+
+_lib = None
+
+
+def load() -> ctypes.CDLL:
+    """Load libscaleqlora.so from the package directory (raises if it was not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2609_04526_gb300.build` "
+                          "(or __graft_entry__.build()); there is no fallback path")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+    W = ctypes.POINTER(_SqWeight)
+    L.sq_create.argtypes = [ctypes.POINTER(vp)]
+    L.sq_destroy.argtypes = [vp]
+    L.sq_status_string.argtypes = [ctypes.c_int]
+    L.sq_status_string.restype = ctypes.c_char_p
+    L.sq_last_error.argtypes = [vp]
+    L.sq_last_error.restype = ctypes.c_char_p
+    L.sq_sync.argtypes = [vp, vp]
+    L.sq_fwd.argtypes = [vp, W, vp, i64, vp, vp]
+    L.sq_bwd_dx.argtypes = [vp, W, vp, i64, vp, vp]
+    L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
+    L.sq_project_scales.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
+    L.sq_merge.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
+    for name in EXPORTS:
+        if name not in ("sq_status_string", "sq_last_error"):
+            getattr(L, name).restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+@dataclasses.dataclass
+class QuantWeight:
+    """One native-FP4 linear, weight [N, K]: packed codes [N, K/2] u8, scales [N, K/B] u8, ws2."""
+    fmt: int
+    N: int
+    K: int
+    codes: torch.Tensor
+    scales: Optional[torch.Tensor]
+    ws2: float
+
+    def _c(self) -> _SqWeight:
+        return _SqWeight(self.fmt, self.N, self.K, _ptr(self.codes), _ptr(self.scales), self.ws2)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+class Handle:
+    """Owns one sq_handle (not thread-safe: one per host thread)."""
+
+    def __init__(self):
+        self._L = load()
+        h = ctypes.c_void_p()
+        st = self._L.sq_create(ctypes.byref(h))
+        if st != SQ_OK:
+            raise SQError(st, "sq_create failed")
+        self._h = h
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._L.sq_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, st: int):
+        if st != SQ_OK:
+            raise SQError(st, self._L.sq_last_error(self._h).decode())
+
+    # raw status variants (no exception) -------------------------------------
+    def status_of(self, name: str, *args) -> int:
+        return getattr(self._L, name)(self._h, *args)
+
+    def last_error(self) -> str:
+        return self._L.sq_last_error(self._h).decode()
+
+    # entry points ------------------------------------------------------------
+    def sq_sync(self, stream=None):
+        self._check(self._L.sq_sync(self._h, _stream(stream)))
+
+    def sq_fwd(self, w: QuantWeight, X: torch.Tensor, Y: Optional[torch.Tensor] = None, stream=None):
+        M = X.shape[0]
+        if Y is None:
+            Y = torch.empty(M, w.N, dtype=torch.bfloat16, device=X.device)
+        wc = w._c()
+        self._check(self._L.sq_fwd(self._h, ctypes.byref(wc), _ptr(X), M, _ptr(Y), _stream(stream)))
+        return Y
+
+    def sq_bwd_dx(self, w: QuantWeight, dY: torch.Tensor, dX: Optional[torch.Tensor] = None, stream=None):
+        M = dY.shape[0]
+        if dX is None:
+            dX = torch.empty(M, w.K, dtype=torch.bfloat16, device=dY.device)
+        wc = w._c()
+        self._check(self._L.sq_bwd_dx(self._h, ctypes.byref(wc), _ptr(dY), M, _ptr(dX), _stream(stream)))
+        return dX
+
+    def sq_scale_grad(self, w: QuantWeight, X: torch.Tensor, dY: torch.Tensor, mask: Optional[torch.Tensor] = None,
+                      g: Optional[torch.Tensor] = None, stream=None):
+        M = X.shape[0]
+        if g is None:
+            g = torch.empty(w.N, w.K // BLOCK[w.fmt], dtype=torch.float32, device=X.device)
+        wc = w._c()
+        self._check(self._L.sq_scale_grad(self._h, ctypes.byref(wc), _ptr(X), _ptr(dY), M, _ptr(mask), _ptr(g),
+                                          _stream(stream)))
+        return g
+
+    def sq_project_scales(self, fmt: int, latent: torch.Tensor, ws2: float, bytes_out: Optional[torch.Tensor] = None,
+                          mask_out: Optional[torch.Tensor] = None, nonfinite: Optional[torch.Tensor] = None,
+                          want_mask: bool = True, stream=None):
+        N, G = latent.shape
+        if bytes_out is None:
+            bytes_out = torch.empty(N, G, dtype=torch.uint8, device=latent.device)
+        if mask_out is None and want_mask:
+            mask_out = torch.empty(N, G, dtype=torch.uint8, device=latent.device)
+        self._check(self._L.sq_project_scales(self._h, fmt, N, G, ws2, _ptr(latent), _ptr(bytes_out), _ptr(mask_out),
+                                              _ptr(nonfinite), _stream(stream)))
+        return bytes_out, mask_out
+
+    def sq_merge(self, fmt: int, latent: torch.Tensor, ws2: float, scales_inout: torch.Tensor,
+                 ongrid_delta: Optional[torch.Tensor] = None, changed: Optional[torch.Tensor] = None, stream=None):
+        N, G = latent.shape
+        self._check(self._L.sq_merge(self._h, fmt, N, G, ws2, _ptr(latent), _ptr(scales_inout), _ptr(ongrid_delta),
+                                     _ptr(changed), _stream(stream)))
+        return scales_inout

@@ -1,0 +1,343 @@
+// Host layer of libscaleqlora: argument validation, device checks, TMA
+// descriptor encoding and kernel launches behind the C ABI of scaleqlora.h.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "scaleqlora.h"
+#include "sq_internal.h"
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+struct DeviceState {
+  int device;
+  int sm_count;
+  int *err_word;  // device int, written by kernels whose bounded waits ran out
+};
+
+constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
+constexpr int64_t kMaxTokens = (int64_t(1) << 31) - 1;  // TMA coordinates are int32
+
+}  // namespace
+
+struct sq_handle_s {
+  std::string last_error;
+  std::vector<DeviceState> devices;
+  EncodeTiledFn encode = nullptr;
+};
+
+namespace {
+
+sq_status fail(sq_handle h, sq_status s, const char *fmt, ...) {
+  if (h) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    h->last_error = buf;
+  }
+  return s;
+}
+
+sq_status cuda_fail(sq_handle h, cudaError_t e, const char *what) {
+  return fail(h, SQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Current device: checked for compute capability 10.3, error word allocated once.
+sq_status ensure_device(sq_handle h, DeviceState **out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(h, SQ_ERR_DEVICE, "no CUDA device: %s", cudaGetErrorString(e));
+  for (auto &d : h->devices)
+    if (d.device == dev) {
+      *out = &d;
+      return SQ_OK;
+    }
+  int major = 0, minor = 0, sms = 0;
+  if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess ||
+      (e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess ||
+      (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return cuda_fail(h, e, "device query");
+  if (major != 10 || minor != 3)
+    return fail(h, SQ_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a only", dev, major,
+                minor);
+  if (!h->encode) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+      return fail(h, SQ_ERR_DEVICE, "driver entry point cuTensorMapEncodeTiled unavailable");
+    h->encode = reinterpret_cast<EncodeTiledFn>(fn);
+  }
+  int *err_word = nullptr;
+  if ((e = cudaMalloc(&err_word, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(error word)");
+  if ((e = cudaMemset(err_word, 0, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(error word)");
+  h->devices.push_back(DeviceState{dev, sms, err_word});
+  *out = &h->devices.back();
+  return SQ_OK;
+}
+
+// 2-D bf16 tensor [outer, inner] (row-major, inner contiguous) loaded in
+// box_inner x box_outer tiles with the 128-byte swizzle; out-of-range elements
+// read as zero.
+sq_status make_map(sq_handle h, CUtensorMap *map, const void *ptr, int64_t inner, int64_t outer, uint32_t box_inner,
+                   uint32_t box_outer) {
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = h->encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(h, SQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return SQ_OK;
+}
+
+int block_of(int fmt) { return fmt == SQ_NVFP4 ? 16 : 32; }
+
+sq_status check_ws2(sq_handle h, int fmt, float ws2) {
+  if (fmt == SQ_NVFP4) {
+    if (!(std::isfinite(ws2) && ws2 > 0.0f)) return fail(h, SQ_ERR_INVALID_ARG, "NVFP4 ws2 must be finite and > 0");
+  } else if (fmt == SQ_MXFP4) {
+    if (ws2 != 1.0f) return fail(h, SQ_ERR_INVALID_ARG, "MXFP4 ws2 must be 1.0");
+  } else {
+    return fail(h, SQ_ERR_INVALID_ARG, "unknown format %d", fmt);
+  }
+  return SQ_OK;
+}
+
+sq_status check_weight(sq_handle h, const sq_weight *w, bool need_scales) {
+  if (!w) return fail(h, SQ_ERR_INVALID_ARG, "weight is NULL");
+  sq_status s = check_ws2(h, w->fmt, w->ws2);
+  if (s != SQ_OK) return s;
+  if (w->N <= 0 || w->N % 8 != 0 || w->N > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "N=%d must be positive, a multiple of 8 and <= 2^24", w->N);
+  if (w->K <= 0 || w->K % 32 != 0 || w->K > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "K=%d must be positive, a multiple of 32 and <= 2^24", w->K);
+  if (!w->codes || !aligned16(w->codes)) return fail(h, SQ_ERR_INVALID_ARG, "codes must be non-NULL and 16-byte aligned");
+  if (need_scales && (!w->scales || !aligned16(w->scales)))
+    return fail(h, SQ_ERR_INVALID_ARG, "scales must be non-NULL and 16-byte aligned");
+  return SQ_OK;
+}
+
+sq_status check_tokens(sq_handle h, int64_t M) {
+  if (M < 0 || M > kMaxTokens) return fail(h, SQ_ERR_INVALID_ARG, "M=%lld out of range [0, 2^31)", (long long)M);
+  return SQ_OK;
+}
+
+sq_status check_buf(sq_handle h, const void *p, const char *name) {
+  if (!p || !aligned16(p)) return fail(h, SQ_ERR_INVALID_ARG, "%s must be non-NULL and 16-byte aligned", name);
+  return SQ_OK;
+}
+
+#define SQ_TRY(expr)                    \
+  do {                                  \
+    sq_status _s = (expr);              \
+    if (_s != SQ_OK) return _s;         \
+  } while (0)
+
+#define SQ_GUARD_BEGIN try {
+#define SQ_GUARD_END                                                             \
+  }                                                                              \
+  catch (...) {                                                                  \
+    return fail(h, SQ_ERR_CUDA, "internal error (host exception)");              \
+  }
+
+sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr, const void *b_ptr, int64_t M,
+                   void *out, const uint8_t *mask, cudaStream_t stream) {
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  CUtensorMap tmA, tmB;
+  std::memset(&tmB, 0, sizeof(tmB));
+  if (mode == sqi::MODE_FWD) {
+    SQ_TRY(make_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));
+  } else if (mode == sqi::MODE_DX) {
+    SQ_TRY(make_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));
+  } else {
+    SQ_TRY(make_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBK));  // dY, MN-major boxes 64(n) x 64(m)
+    SQ_TRY(make_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kBK));  // X,  MN-major boxes 64(k) x 64(m)
+  }
+  sqi::GemmArgs a;
+  a.mode = mode;
+  a.fmt = w->fmt;
+  a.M = M;
+  a.N = w->N;
+  a.K = w->K;
+  a.codes = w->codes;
+  a.scales = w->scales;
+  a.ws2 = w->ws2;
+  a.out = out;
+  a.mask = mask;
+  a.err = dev->err_word;
+  cudaError_t e = sqi::launch_gemm(a, tmA, tmB, dev->sm_count, stream);
+  if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
+  return SQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+sq_status sq_create(sq_handle *out) {
+  if (!out) return SQ_ERR_INVALID_ARG;
+  try {
+    *out = new sq_handle_s();
+  } catch (...) {
+    *out = nullptr;
+    return SQ_ERR_CUDA;
+  }
+  return SQ_OK;
+}
+
+sq_status sq_destroy(sq_handle h) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  int cur = -1;
+  cudaGetDevice(&cur);
+  for (auto &d : h->devices) {
+    if (cudaSetDevice(d.device) == cudaSuccess) cudaFree(d.err_word);
+  }
+  if (cur >= 0) cudaSetDevice(cur);
+  delete h;
+  return SQ_OK;
+}
+
+const char *sq_status_string(sq_status s) {
+  switch (s) {
+    case SQ_OK: return "SQ_OK";
+    case SQ_ERR_INVALID_ARG: return "SQ_ERR_INVALID_ARG";
+    case SQ_ERR_UNSUPPORTED: return "SQ_ERR_UNSUPPORTED";
+    case SQ_ERR_DEVICE: return "SQ_ERR_DEVICE";
+    case SQ_ERR_CUDA: return "SQ_ERR_CUDA";
+    case SQ_ERR_DEVICE_TIMEOUT: return "SQ_ERR_DEVICE_TIMEOUT";
+  }
+  return "SQ_ERR_UNKNOWN";
+}
+
+const char *sq_last_error(sq_handle h) { return h ? h->last_error.c_str() : "NULL handle"; }
+
+sq_status sq_sync(sq_handle h, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamSynchronize");
+  int dev = -1;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail(h, e, "cudaGetDevice");
+  for (auto &d : h->devices) {
+    if (d.device != dev) continue;
+    int word = 0;
+    if ((e = cudaMemcpy(&word, d.err_word, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+      return cuda_fail(h, e, "reading the device error word");
+    if (word != 0) {
+      cudaMemset(d.err_word, 0, sizeof(int));
+      return fail(h, SQ_ERR_DEVICE_TIMEOUT, "a bounded device wait ran out (error word 0x%x)", word);
+    }
+  }
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_fwd(sq_handle h, const sq_weight *w, const uint16_t *X, int64_t M, uint16_t *Y, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_weight(h, w, true));
+  SQ_TRY(check_tokens(h, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, Y, "Y"));
+  return run_gemm(h, sqi::MODE_FWD, w, X, nullptr, M, Y, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_bwd_dx(sq_handle h, const sq_weight *w, const uint16_t *dY, int64_t M, uint16_t *dX, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_weight(h, w, true));
+  SQ_TRY(check_tokens(h, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, dY, "dY"));
+  SQ_TRY(check_buf(h, dX, "dX"));
+  return run_gemm(h, sqi::MODE_DX, w, dY, nullptr, M, dX, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
+                        const uint8_t *mask, float *g, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_weight(h, w, false));
+  SQ_TRY(check_tokens(h, M));
+  SQ_TRY(check_buf(h, g, "g"));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (M == 0) {
+    DeviceState *dev = nullptr;
+    SQ_TRY(ensure_device(h, &dev));
+    const size_t bytes = static_cast<size_t>(w->N) * (w->K / block_of(w->fmt)) * sizeof(float);
+    cudaError_t e = cudaMemsetAsync(g, 0, bytes, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(g)");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, dY, "dY"));
+  return run_gemm(h, sqi::MODE_SGRAD, w, dY, X, M, g, mask, st);
+  SQ_GUARD_END
+}
+
+static sq_status check_plane(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2) {
+  SQ_TRY(check_ws2(h, fmt, ws2));
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  return SQ_OK;
+}
+
+sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
+                            uint8_t *bytes_out, uint8_t *mask_out, int32_t *nonfinite, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_plane(h, fmt, N, G, ws2));
+  SQ_TRY(check_buf(h, latent, "latent"));
+  SQ_TRY(check_buf(h, bytes_out, "bytes_out"));
+  if (mask_out && !aligned16(mask_out)) return fail(h, SQ_ERR_INVALID_ARG, "mask_out must be 16-byte aligned");
+  if (nonfinite && (reinterpret_cast<uintptr_t>(nonfinite) & 3u))
+    return fail(h, SQ_ERR_INVALID_ARG, "nonfinite must be 4-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_project(fmt, N * G, ws2, latent, bytes_out, mask_out, nonfinite, dev->sm_count,
+                                      static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
+                   uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_plane(h, fmt, N, G, ws2));
+  SQ_TRY(check_buf(h, latent, "latent"));
+  SQ_TRY(check_buf(h, scales_inout, "scales_inout"));
+  if (ongrid_delta && !aligned16(ongrid_delta)) return fail(h, SQ_ERR_INVALID_ARG, "ongrid_delta must be 16-byte aligned");
+  if (changed_bytes && (reinterpret_cast<uintptr_t>(changed_bytes) & 7u))
+    return fail(h, SQ_ERR_INVALID_ARG, "changed_bytes must be 8-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_merge(fmt, N * G, ws2, latent, scales_inout, ongrid_delta, changed_bytes, dev->sm_count,
+                                    static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+}  // extern "C"

@@ -1,0 +1,50 @@
+// Internal declarations shared by the host layer (sq_api.cu) and the kernel
+// translation units of libscaleqlora. Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace sqi {
+
+enum GemmMode : int {
+  MODE_FWD = 0,    // Y  = X  . W^T   (GEMM M=tokens, N=out, contraction=in)
+  MODE_DX = 1,     // dX = dY . W     (GEMM M=tokens, N=in,  contraction=out)
+  MODE_SGRAD = 2   // g  = blockreduce(code * dY^T X)  (GEMM M=out, N=in, contraction=tokens)
+};
+
+// Tile shape of the tcgen05 contraction kernels: one 128 x 256 fp32
+// accumulator in TMEM per CTA, 64-deep k-steps through a 4-stage smem ring.
+constexpr int kBM = 128;
+constexpr int kBN = 256;
+constexpr int kBK = 64;
+constexpr int kStages = 4;
+
+struct GemmArgs {
+  int mode;
+  int fmt;               // 0 NVFP4, 1 MXFP4
+  int64_t M, N, K;       // tokens, out features, in features
+  const uint8_t *codes;  // [N, K/2]
+  const uint8_t *scales; // [N, K/B]
+  float ws2;
+  void *out;             // Y [M,N] bf16 | dX [M,K] bf16 | g [N,K/B] f32
+  const uint8_t *mask;   // [N, K/B] or null (MODE_SGRAD only)
+  int *err;              // device error word
+};
+
+// Launch one contraction. tmA / tmB are the TMA descriptors of the streamed
+// bf16 operands (tmB is used by MODE_SGRAD only).
+cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
+                        cudaStream_t stream);
+
+cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *latent, uint8_t *bytes_out,
+                           uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream);
+
+cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *scales_inout,
+                         float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream);
+
+// Device-side error codes written to the error word.
+constexpr int kErrWaitTimeout = 1;
+
+}  // namespace sqi

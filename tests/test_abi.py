@@ -1,0 +1,105 @@
+"""The C-ABI library loads without a GPU, exports every entry point the header
+declares, and rejects bad arguments before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+pkg = pytest.importorskip("paper_2609_04526_gb300")
+
+
+@pytest.fixture(scope="module")
+def built():
+    from paper_2609_04526_gb300 import build
+    build.build()
+    return pkg.load()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "scaleqlora.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(sq_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(built):
+    declared = _declared()
+    assert set(declared) == set(pkg._lib.EXPORTS)
+    for name in declared:
+        assert hasattr(built, name), name
+
+
+def test_status_strings(built):
+    for code, name in pkg._lib.STATUS.items():
+        assert built.sq_status_string(code).decode() == name
+    assert built.sq_status_string(7).decode() == "SQ_ERR_UNKNOWN"
+
+
+def test_null_handle_and_create(built):
+    assert built.sq_fwd(None, None, None, 0, None, None) == -1
+    assert built.sq_create(None) == -1
+    h = pkg.Handle()
+    h.close()
+
+
+A16 = 0x10000  # a 16-byte aligned address that is never dereferenced (validation fails first)
+
+
+def _w(fmt=0, N=256, K=512, codes=A16, scales=A16, ws2=0.01):
+    return pkg._lib._SqWeight(fmt, N, K, codes, scales, ws2)
+
+
+@pytest.mark.parametrize("w, why", [
+    (None, "weight is NULL"),
+    (_w(fmt=2), "unknown format"),
+    (_w(N=0), "N=0"),
+    (_w(N=12), "N=12"),
+    (_w(K=48), "K=48"),
+    (_w(K=-32), "K=-32"),
+    (_w(codes=0), "codes"),
+    (_w(codes=A16 + 8), "codes"),
+    (_w(scales=0), "scales"),
+    (_w(ws2=0.0), "ws2"),
+    (_w(ws2=float("nan")), "ws2"),
+    (_w(fmt=1, ws2=0.5), "MXFP4 ws2"),
+])
+def test_weight_validation(built, w, why):
+    h = pkg.Handle()
+    wp = ctypes.byref(w) if w is not None else None
+    assert h.status_of("sq_fwd", wp, ctypes.c_void_p(A16), 4, ctypes.c_void_p(A16), None) == -1
+    assert why.split("=")[0].split()[0] in h.last_error()
+
+
+def test_buffer_and_token_validation(built):
+    h = pkg.Handle()
+    w = _w()
+    vp = ctypes.c_void_p
+    assert h.status_of("sq_fwd", ctypes.byref(w), vp(A16), -1, vp(A16), None) == -1
+    assert h.status_of("sq_fwd", ctypes.byref(w), vp(A16), 1 << 31, vp(A16), None) == -1
+    assert h.status_of("sq_fwd", ctypes.byref(w), vp(A16 + 2), 4, vp(A16), None) == -1
+    assert h.status_of("sq_bwd_dx", ctypes.byref(w), vp(A16), 4, None, None) == -1
+    assert h.status_of("sq_scale_grad", ctypes.byref(w), vp(A16), vp(A16), 4, None, None, None) == -1
+    assert h.status_of("sq_project_scales", 0, 4, 16, 0.0, vp(A16), vp(A16), None, None, None) == -1
+    assert h.status_of("sq_project_scales", 0, 4, 16, 1.0, vp(A16), vp(A16 + 1), None, None, None) == -1
+    assert h.status_of("sq_project_scales", 1, 4, 16, 2.0, vp(A16), vp(A16), None, None, None) == -1
+    assert h.status_of("sq_merge", 0, -1, 16, 1.0, vp(A16), vp(A16), None, None, None) == -1
+    assert h.status_of("sq_merge", 0, 4, 16, 1.0, vp(A16), vp(A16), vp(A16 + 4), None, None) == -1
+
+
+def test_empty_batch_is_a_noop_without_device(built):
+    """M == 0 for the forward / input gradient enqueues nothing."""
+    h = pkg.Handle()
+    w = _w()
+    assert h.status_of("sq_fwd", ctypes.byref(w), None, 0, None, None) == 0
+    assert h.status_of("sq_bwd_dx", ctypes.byref(w), None, 0, None, None) == 0
+
+
+def test_binding_refuses_to_fall_back(tmp_path, monkeypatch):
+    """Without the shared library the binding raises instead of computing elsewhere."""
+    import paper_2609_04526_gb300._lib as L
+    monkeypatch.setattr(L, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(L, "_lib", None)
+    with pytest.raises(ImportError):
+        L.load()

@@ -1,0 +1,234 @@
+"""GPU parity of the five C-ABI entry points against the float64 oracle.
+
+Small shapes (several tiles each, with ragged tails in every dimension) are
+compared element by element over the whole output; the full-size workloads
+are compared on seeded samples the oracle computes one by one, and their
+projected / merged planes bit for bit over every byte."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import assert_close, f64, hbits, host, setup_linear
+
+pytestmark = pytest.mark.gpu
+
+NV, MX = 0, 1
+
+
+@pytest.fixture(scope="module")
+def h():
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+    return pkg.Handle()
+
+
+SMALL = [
+    # key, fmt, M, N, K      (tiles are 128 x 256 with 64-deep k-steps)
+    ("c1", NV, 64, 256, 512),
+    ("nv_ragged", NV, 300, 392, 608),
+    ("mx_ragged", MX, 257, 264, 544),
+    ("nv_min", NV, 1, 8, 32),
+    ("mx_min", MX, 3, 8, 32),
+    ("mx_tall", MX, 1000, 520, 96),
+    ("nv_long_k", NV, 70, 136, 2080),
+    ("nv_long_m", NV, 1500, 40, 256),
+]
+
+
+def _wl(key, fmt, M, N, K):
+    from paper_2609_04526_gb300 import synth
+    if key in synth.WORKLOADS:
+        return synth.WORKLOADS[key]
+    return synth.custom(key, fmt, M, N, K, seed=abs(hash((fmt, M, N, K))) % 10000, kind="outlier" if fmt else "gauss")
+
+
+@pytest.mark.parametrize("key,fmt,M,N,K", SMALL, ids=[s[0] for s in SMALL])
+def test_full_parity_small(h, key, fmt, M, N, K):
+    wl = _wl(key, fmt, M, N, K)
+    lin = wl.linears[0]
+    w, X, dY = setup_linear(wl, lin)
+    assert (w.N, w.K, X.shape[0]) == (N, K, M)
+    rng = np.random.default_rng(M * 7 + N)
+    G = K // (16 if fmt == NV else 32)
+    mask = torch.from_numpy(rng.integers(0, 2, size=(N, G), dtype=np.uint8)).cuda()
+    Y = h.sq_fwd(w, X)
+    dX = h.sq_bwd_dx(w, dY)
+    g = h.sq_scale_grad(w, X, dY)
+    gm = h.sq_scale_grad(w, X, dY, mask=mask)
+    h.sq_sync()
+    codes, scales = host(w.codes), host(w.scales)
+    Y_ref = oracle.fwd(fmt, codes, scales, w.ws2, hbits(X))
+    dX_ref = oracle.dx(fmt, codes, scales, w.ws2, hbits(dY))
+    g_ref = oracle.scale_grad(fmt, codes, hbits(X), hbits(dY))
+    assert_close(f64(Y), Y_ref, what="Y")
+    assert_close(f64(dX), dX_ref, what="dX")
+    assert_close(f64(g), g_ref, what="g")
+    assert_close(f64(gm), g_ref * host(mask), rms=float(np.sqrt(np.mean(g_ref ** 2))), what="g*mask")
+
+
+def _sampled_checks(h, wl, lin, n_samples=4096, n_rows=32):
+    w, X, dY = setup_linear(wl, lin)
+    codes0 = w.codes.clone()
+    Y = h.sq_fwd(w, X)
+    dX = h.sq_bwd_dx(w, dY)
+    g = h.sq_scale_grad(w, X, dY)
+    h.sq_sync()
+    M, N, K = X.shape[0], w.N, w.K
+    rng = np.random.default_rng(wl.seed)
+    ms = rng.integers(0, M, n_samples)
+    ns = rng.integers(0, N, n_samples)
+    ks = rng.integers(0, K, n_samples)
+    # always include the corners of the last (ragged or not) tiles
+    ms[:4] = [0, M - 1, 0, M - 1]
+    ns[:4] = [0, 0, N - 1, N - 1]
+    ks[:4] = [0, 0, K - 1, K - 1]
+    codes, scales = host(w.codes), host(w.scales)
+    Xb, dYb = hbits(X), hbits(dY)
+    Yh, dXh, gh = f64(Y), f64(dX), f64(g)
+    Y_ref = oracle.fwd_at(wl.fmt, codes, scales, w.ws2, Xb, ms, ns)
+    dX_ref = oracle.dx_at(wl.fmt, codes, scales, w.ws2, dYb, ms, ks)
+    assert_close(Yh[ms, ns], Y_ref, what=f"{wl.key}/{lin.name} Y samples")
+    assert_close(dXh[ms, ks], dX_ref, what=f"{wl.key}/{lin.name} dX samples")
+    rows = np.unique(np.concatenate([[0, N - 1], rng.integers(0, N, n_rows)]))
+    g_ref = oracle.scale_grad(wl.fmt, codes, Xb, dYb, rows=rows)
+    assert_close(gh[rows], g_ref, what=f"{wl.key}/{lin.name} g rows")
+    assert torch.equal(w.codes, codes0)
+    return w
+
+
+@pytest.mark.parametrize("key", ["c2", "c3", "c4"])
+def test_sampled_parity_full_size(h, key):
+    from paper_2609_04526_gb300 import synth
+    wl = synth.WORKLOADS[key]
+    _sampled_checks(h, wl, wl.linears[0])
+    torch.cuda.empty_cache()
+
+
+def test_layer_step_and_merge_c5(h):
+    """The 7-linear decoder layer at 16 x 2048 tokens: sampled parity for two
+    linears of different shape, then projection and merge of all 7 scale planes
+    bit-exact against the oracle, with every code plane byte-identical."""
+    from paper_2609_04526_gb300 import synth
+    wl = synth.WORKLOADS["c5"]
+    by_name = {l.name: l for l in wl.linears}
+    for name in ("k_proj", "down_proj"):
+        _sampled_checks(h, wl, by_name[name], n_samples=2048, n_rows=8)
+        torch.cuda.empty_cache()
+    total_changed = 0
+    for lin in wl.linears:
+        w = synth.gen_weight(wl, lin, device="cuda")
+        codes_before = w.codes.clone()
+        L = synth.gen_latent(wl, lin, w, device="cuda")
+        nf = torch.zeros(1, dtype=torch.int32, device="cuda")
+        b, m = h.sq_project_scales(wl.fmt, L, w.ws2, nonfinite=nf)
+        scales = w.scales.clone()
+        delta = torch.empty_like(L)
+        ch = torch.zeros(1, dtype=torch.int64, device="cuda")
+        h.sq_merge(wl.fmt, L, w.ws2, scales, ongrid_delta=delta, changed=ch)
+        h.sq_sync()
+        Lh = host(L)
+        rb, rm, rnf = oracle.project(wl.fmt, Lh, w.ws2)
+        rs, rd, rch = oracle.merge(wl.fmt, Lh, host(w.scales), w.ws2)
+        assert np.array_equal(host(b), rb) and np.array_equal(host(m), rm) and int(nf.item()) == rnf
+        assert np.array_equal(host(scales), rs) and int(ch.item()) == rch
+        dh = host(delta)
+        assert np.array_equal(np.isnan(dh), np.isnan(rd))
+        assert np.array_equal(dh.view(np.uint32)[~np.isnan(dh)], rd.view(np.uint32)[~np.isnan(rd)])
+        assert torch.equal(w.codes, codes_before)
+        total_changed += rch
+    frac = total_changed / sum(l.N * l.K // wl.block for l in wl.linears)
+    assert 0.005 < frac < 0.2, frac
+
+
+def _edge_latents(fmt, ws2):
+    rng = np.random.default_rng(99)
+    vals = []
+    if fmt == NV:
+        grid = torch.arange(256, dtype=torch.uint8).view(torch.float8_e4m3fn).float().numpy()
+        pos = grid[1:0x7F].astype(np.float64)
+        mids = (pos[:-1] + pos[1:]) / 2
+        cap = np.float32(448.0) * np.float32(ws2)
+        vals += list(pos * ws2) + list(mids * ws2) + list(-mids * ws2)
+        vals += [cap, np.nextafter(cap, np.float32(1e30)), cap * 2, -cap, -cap * 3]
+        vals += [2.0 ** -10 * ws2, 2.0 ** -11 * ws2, 1e-30, -1e-30]
+    else:
+        e = np.arange(-130, 130)
+        vals += list(np.ldexp(1.0, e)) + list(np.ldexp(np.sqrt(2.0), e)) + list(np.ldexp(1.4142135, e))
+        vals += list(np.ldexp(1.4142137, e)) + [2.0 ** -149, 3e-45, 1.5 * 2.0 ** 127, 3.4e38, -1.0]
+    vals += [0.0, -0.0, np.inf, -np.inf, np.nan, -np.nan]
+    vals += list(rng.standard_normal(1000) * (ws2 if fmt == NV else 1e-3))
+    a = np.array(vals, dtype=np.float32)
+    return a  # length not a multiple of 16 on purpose
+
+
+@pytest.mark.parametrize("fmt,ws2", [(NV, 1.0), (NV, 0.0123), (NV, 2.0 ** -9), (MX, 1.0)])
+def test_projection_and_merge_edges_bit_exact(h, fmt, ws2):
+    ws2 = float(np.float32(ws2))
+    L = _edge_latents(fmt, ws2)
+    n = L.size
+    for count in (n, n - 5, 17, 16, 15, 1):
+        Lc = L[:count].reshape(1, count)
+        Ld = torch.from_numpy(Lc.copy()).cuda()
+        nf = torch.full((1,), 77, dtype=torch.int32, device="cuda")
+        b, m = h.sq_project_scales(fmt, Ld, ws2, nonfinite=nf)
+        old = torch.from_numpy(np.random.default_rng(count).integers(0, 0x7F if fmt == NV else 255, size=(1, count),
+                                                                      dtype=np.uint8)).cuda()
+        sc = old.clone()
+        delta = torch.empty_like(Ld)
+        ch = torch.full((1,), 5, dtype=torch.int64, device="cuda")
+        h.sq_merge(fmt, Ld, ws2, sc, ongrid_delta=delta, changed=ch)
+        h.sq_sync()
+        rb, rm, rnf = oracle.project(fmt, Lc, ws2)
+        assert np.array_equal(host(b), rb), np.nonzero(host(b) != rb)
+        assert np.array_equal(host(m), rm)
+        assert int(nf.item()) == rnf
+        rs, rd, rch = oracle.merge(fmt, Lc, host(old), ws2)
+        assert np.array_equal(host(sc), rs) and int(ch.item()) == rch
+        dh = host(delta)
+        assert np.array_equal(np.isnan(dh), np.isnan(rd))
+        ok = ~np.isnan(rd)
+        assert np.array_equal(dh.view(np.uint32)[ok], rd.view(np.uint32)[ok])
+
+
+def test_projection_dense_sweep_bit_exact(h):
+    """2^24 latents spread over the whole E4M3 range (and past the ceiling) and a
+    full fp32 binade for E8M0: every byte and mask bit equals the oracle's."""
+    rng = np.random.default_rng(7)
+    ws2 = float(np.float32(0.00731))
+    L = (np.exp(rng.uniform(np.log(1e-7), np.log(600), size=1 << 24)) * rng.choice([-1, 1], size=1 << 24) * ws2)
+    L = L.astype(np.float32).reshape(1 << 12, 1 << 12)
+    b, m = h.sq_project_scales(NV, torch.from_numpy(L).cuda(), ws2)
+    rb, rm, _ = oracle.project(NV, L, ws2)
+    assert np.array_equal(host(b), rb) and np.array_equal(host(m), rm)
+    j = np.arange(1 << 23, dtype=np.int64)
+    Lm = (1.0 + j / float(1 << 23)).astype(np.float32).reshape(1 << 11, 1 << 12) * np.float32(2.0 ** -20)
+    b, m = h.sq_project_scales(MX, torch.from_numpy(Lm).cuda(), 1.0)
+    rb, rm, _ = oracle.project(MX, Lm, 1.0)
+    assert np.array_equal(host(b), rb) and np.array_equal(host(m), rm)
+
+
+def test_empty_batch_and_sync(h):
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom("e", NV, 4, 64, 128, seed=1)
+    w, X, dY = setup_linear(wl, wl.linears[0])
+    g = torch.full((64, 8), 3.0, device="cuda")
+    h.sq_scale_grad(w, X[:0], dY[:0], g=g)
+    Y = torch.full((0, 64), 1.0, dtype=torch.bfloat16, device="cuda")
+    h.sq_fwd(w, X[:0], Y)
+    h.sq_sync()
+    assert (g == 0).all()
+
+
+def test_invalid_args_on_device(h):
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom("e", NV, 4, 64, 128, seed=2)
+    w, X, dY = setup_linear(wl, wl.linears[0])
+    bad = pkg.QuantWeight(w.fmt, 60, w.K, w.codes, w.scales, w.ws2)
+    with pytest.raises(pkg.SQError):
+        h.sq_fwd(bad, X)
+    with pytest.raises(pkg.SQError):
+        h.sq_fwd(w, X[:, 1:])  # misaligned base
