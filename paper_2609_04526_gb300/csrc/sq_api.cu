@@ -90,20 +90,26 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   return SQ_OK;
 }
 
-// 2-D bf16 tensor [outer, inner] (row-major, inner contiguous) loaded in
-// box_inner x box_outer tiles with the 128-byte swizzle; out-of-range elements
-// read as zero.
-sq_status make_map(sq_handle h, CUtensorMap *map, const void *ptr, int64_t inner, int64_t outer, uint32_t box_inner,
-                   uint32_t box_outer) {
+// 2-D tensor [outer, inner] (row-major, inner contiguous) loaded in
+// box_inner x box_outer tiles; out-of-range elements read as zero.
+sq_status make_map(sq_handle h, CUtensorMap *map, const void *ptr, CUtensorMapDataType dtype, int elem_bytes,
+                   int64_t inner, int64_t outer, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * elem_bytes};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  CUresult r = h->encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = h->encode(map, dtype, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(h, SQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
   return SQ_OK;
+}
+
+// bf16 activation tensor with the 128-byte swizzle the MMA descriptors expect.
+sq_status make_act_map(sq_handle h, CUtensorMap *map, const void *ptr, int64_t inner, int64_t outer,
+                       uint32_t box_inner, uint32_t box_outer) {
+  return make_map(h, map, ptr, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, inner, outer, box_inner, box_outer,
+                  CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 int block_of(int fmt) { return fmt == SQ_NVFP4 ? 16 : 32; }
@@ -161,14 +167,20 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   DeviceState *dev = nullptr;
   SQ_TRY(ensure_device(h, &dev));
   CUtensorMap tmA, tmB;
-  std::memset(&tmB, 0, sizeof(tmB));
+  const int64_t K2 = w->K / 2;  // code bytes per row
   if (mode == sqi::MODE_FWD) {
-    SQ_TRY(make_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));  // X, 128 x 64 K-major boxes
+    // codes: 256 rows x 32 bytes (64 weights) per k-step
+    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, sqi::kBK / 2, sqi::kBN,
+                    CU_TENSOR_MAP_SWIZZLE_NONE));
   } else if (mode == sqi::MODE_DX) {
-    SQ_TRY(make_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));  // dY, 128 x 64 K-major boxes
+    // codes: 64 contraction rows x 128 bytes (256 weights) per k-step, 128-byte swizzle
+    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, sqi::kBN / 2, sqi::kBK,
+                    CU_TENSOR_MAP_SWIZZLE_128B));
   } else {
-    SQ_TRY(make_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBK));  // dY, MN-major boxes 64(n) x 64(m)
-    SQ_TRY(make_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kBK));  // X,  MN-major boxes 64(k) x 64(m)
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBK));  // dY, MN-major boxes 64(n) x 64(m)
+    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kBK));  // X,  MN-major boxes 64(k) x 64(m)
   }
   sqi::GemmArgs a;
   a.mode = mode;

@@ -4,17 +4,21 @@
 //   MODE_DX    dX[m,k] = sum_n dY[m,n] W[n,k]       its input gradient
 //   MODE_SGRAD g[n,b]  = sum_{k in b} code[n,k] sum_m dY[m,n] X[m,k]   its scale gradient
 //
-// with W[n,k] = code[n,k] * s[n, k/B] (Sec. 2). One CTA owns one 128 x 256 fp32
-// accumulator tile in tensor memory (TMEM) and runs warp-specialised roles:
-//   warps 0-3  decode (FWD/DX): packed E2M1 nibbles x scale byte -> bf16 operand
-//              tile written straight into the 128B-swizzled smem layout the
-//              tensor core reads; then the epilogue (TMEM -> registers -> HBM).
-//   warp 4     TMA producer: streams the bf16 activation tiles into a 4-stage ring.
-//   warp 5     TMEM allocator and the single MMA-issuing thread (tcgen05.mma,
-//              kind::f16 with bf16 operands, fp32 accumulation).
+// with W[n,k] = code[n,k] * s[n, k/B] (Sec. 2). Persistent CTAs (one per SM)
+// walk 128 x 256 output tiles in an L2-friendly grouped order. Each tile
+// accumulates in one of two 256-column fp32 buffers in tensor memory (TMEM),
+// so the epilogue of one tile overlaps the mainloop of the next. Roles:
+//   warps 0-3   epilogue: tcgen05.ld (one TMEM lane = one output row per thread),
+//               ws2 scaling and bf16 stores (FWD/DX); code x dW products summed
+//               per block, mask, fp32 stores (SGRAD) -- dW never reaches HBM.
+//   warps 4-11  (FWD/DX) decode: the TMA-staged packed-code tile plus the scale
+//               bytes -> bf16 operand tile written straight into the 128B-swizzled
+//               smem layout the tensor core reads (K-major for FWD, MN-major for DX).
+//   next warp   TMA producer: activation tiles (and code tiles) into a 4-stage ring.
+//   last warp   TMEM allocator and the single MMA-issuing thread (tcgen05.mma,
+//               kind::f16, bf16 operands, fp32 accumulation).
 // For MODE_SGRAD both operands are MN-major TMA tiles (dY^T and X, contraction
-// over tokens); the epilogue multiplies each dW element by its code and sums
-// every block of B columns in registers, so dW never reaches HBM.
+// over tokens) and there are no decode warps.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA records
 // kErrWaitTimeout in the device error word, stops issuing, drains what it has
@@ -28,12 +32,9 @@
 namespace sqi {
 namespace {
 
-constexpr int kThreads = 192;
-constexpr int kDecodeWarps = 4;
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemCols = 256;          // one accumulator buffer (two are allocated)
 constexpr int kAStageBytes = kBM * kBK * 2;  // 16 KiB
 constexpr int kBStageBytes = kBN * kBK * 2;  // 32 KiB
-constexpr int kSmemBytes = kStages * (kAStageBytes + kBStageBytes) + 1024 /*align*/ + 256 /*barriers*/;
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s
 
 // ---------------------------------------------------------------- PTX helpers
@@ -244,14 +245,17 @@ __device__ __forceinline__ void e2m1x8_to_bf16(uint32_t w, uint32_t (&o)[4]) {
 }
 
 // Scale byte -> bf16 value replicated in both halves (exact: E4M3 has 4
-// significant bits, E8M0 is a power of two).
+// significant bits, E8M0 is a power of two). E4M3: the 7 magnitude bits placed
+// at fp32 bit 20 read as E4M3(byte) * 2^-120 for normal and subnormal bytes
+// alike, so one multiply by 2^120 gives the value; byte 0x7F / 0xFF is NaN.
 template <int FMT>
 __device__ __forceinline__ uint32_t scale_bf16x2(uint32_t byte) {
   uint32_t u;
   if (FMT == 0) {
-    const __half_raw hr = __nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(byte), __NV_E4M3);
-    const float f = __half2float(__half(hr));
-    u = __bfloat16_as_ushort(__float2bfloat16_rn(f));
+    const uint32_t mag = byte & 0x7Fu;
+    const float f = __uint_as_float(mag << 20) * 0x1p120f;
+    u = (__float_as_uint(f) >> 16) | ((byte & 0x80u) << 8);
+    if (mag == 0x7Fu) u = 0x7FC0u;
   } else {
     u = byte == 0 ? 0x0040u : (byte == 255 ? 0x7FC0u : (byte << 7));
   }
@@ -268,186 +272,255 @@ struct KParams {
   void *out;
   const uint8_t *mask;
   int *err;
+  int tiles_m, tiles_n;
 };
 
+template <int MODE>
+struct Cfg {
+  static constexpr bool kDecode = MODE != MODE_SGRAD;
+  static constexpr int kEpiWarps = 4;                      // warps 0-3: TMEM lanes 0-127
+  static constexpr int kDecWarps = kDecode ? 8 : 0;        // warps 4-11
+  static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
+  static constexpr int kMmaWarp = kTmaWarp + 1;
+  static constexpr int kThreads = 32 * (kMmaWarp + 1);
+  static constexpr int kCStageBytes = kDecode ? 8192 : 0;  // packed-code tile (256 x 64 or 64 x 256 nibbles)
+  static constexpr int kStageBytes = kAStageBytes + kBStageBytes + kCStageBytes;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+  static constexpr uint32_t kTxBytes =
+      MODE == MODE_SGRAD ? kAStageBytes + kBStageBytes : kAStageBytes + kCStageBytes;
+};
+
+// Persistent tile order: tiles are walked in groups of kGroup row-tiles, the
+// column index varying slowest inside a group, so the CTAs resident at any
+// moment share a few row panels and column panels in L2.
+constexpr int kGroup = 8;
+
+__device__ __forceinline__ void tile_coords(int id, int tiles_m, int tiles_n, int &tm, int &tn) {
+  const int per_group = kGroup * tiles_n;
+  const int g = id / per_group;
+  const int first = g * kGroup;
+  const int gm = min(kGroup, tiles_m - first);
+  const int local = id - g * per_group;
+  tm = first + local % gm;
+  tn = local / gm;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+  return v;
+}
+
+// Scale byte(s) covering the 32 weights of one decode unit: two E4M3 bytes
+// (blocks of 16) or one E8M0 byte. Units outside the weight read scale 0; their
+// codes are zero-filled by TMA.
+template <int FMT>
+__device__ __forceinline__ uint32_t load_unit_scale(const KParams &p, int64_t n, int64_t k) {
+  if (n >= p.N || k >= p.K) return 0u;
+  const int64_t G = p.K / (FMT == 0 ? 16 : 32);
+  if (FMT == 0) return __ldg(reinterpret_cast<const unsigned short *>(p.scales + n * G + k / 16));
+  return __ldg(p.scales + n * G + k / 32);
+}
+
+// Weight coordinates (n, k) of decode unit u (0..511) of a k-step.
+template <int MODE>
+__device__ __forceinline__ void unit_coords(int u, int64_t col0, int kb, int64_t &n, int64_t &k) {
+  if (MODE == MODE_FWD) {  // 256 rows (out features) x 64 k: unit = half a row
+    n = col0 + (u >> 1);
+    k = static_cast<int64_t>(kb) * kBK + 32 * (u & 1);
+  } else {  // 64 contraction rows (out features) x 256 k: unit = an eighth of a row
+    n = static_cast<int64_t>(kb) * kBK + (u & 7) + 8 * (u >> 6);
+    k = col0 + 32 * ((u >> 3) & 7);
+  }
+}
+
 template <int MODE, int FMT>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     sq_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const KParams p) {
-  constexpr int B = FMT == 0 ? 16 : 32;
+  using C = Cfg<MODE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t *sA = smem;
-  uint8_t *sB = smem + kStages * kAStageBytes;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(sB + kStages * kBStageBytes);
-  uint64_t *afull = bars;                  // TMA tiles landed        (1 arrival + tx)
-  uint64_t *bfull = bars + kStages;        // decoded B tile written  (kDecodeWarps arrivals)
-  uint64_t *empty = bars + 2 * kStages;    // MMAs reading the stage completed (tcgen05.commit)
-  uint64_t *tfull = bars + 3 * kStages;    // accumulator complete
-  uint64_t *drain = bars + 3 * kStages + 1;
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 3 * kStages + 2);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * C::kStageBytes);
+  uint64_t *afull = bars;                 // TMA tiles of the stage landed      (1 arrival + tx)
+  uint64_t *bfull = bars + kStages;       // decoded B tile written             (kDecWarps arrivals)
+  uint64_t *empty = bars + 2 * kStages;   // MMAs reading the stage completed   (tcgen05.commit)
+  uint64_t *tfull = bars + 3 * kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
+  uint64_t *tempty = tfull + 2;           // [2] accumulator buffer drained     (kEpiWarps arrivals)
+  uint64_t *drain = tempty + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-
-  // GEMM view: rows (TMEM lanes) x cols (TMEM columns), contraction Kg.
-  const int64_t row0 = static_cast<int64_t>(blockIdx.x) * kBM;
-  const int64_t col0 = static_cast<int64_t>(blockIdx.y) * kBN;
-  const int64_t Mg = MODE == MODE_SGRAD ? p.N : p.M;
-  const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
+  const int total = p.tiles_m * p.tiles_n;
   const int64_t Kg = MODE == MODE_FWD ? p.K : (MODE == MODE_DX ? p.N : p.M);
   const int num_k = static_cast<int>((Kg + kBK - 1) / kBK);
+
+  auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
+  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + kAStageBytes; };
+  auto stage_c = [&](int s) { return smem + s * C::kStageBytes + kAStageBytes + kBStageBytes; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&afull[s], 1);
-      mbar_init(&bfull[s], kDecodeWarps);
+      mbar_init(&bfull[s], C::kDecWarps > 0 ? C::kDecWarps : 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(tfull, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], C::kEpiWarps);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 5) tmem_alloc(tmem_slot, kTmemCols);
-  if (warp == 4 && lane == 0) {
+  if (warp == C::kMmaWarp) tmem_alloc(tmem_slot, 2 * kTmemCols);
+  if (warp == C::kTmaWarp && lane == 0) {
     tma_prefetch_desc(&tmA);
-    if (MODE == MODE_SGRAD) tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmB);
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  if (warp == 4) {
+  if (warp == C::kTmaWarp) {
     // ------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int issued = 0;
-      for (int it = 0; it < num_k; ++it) {
-        const int s = it % kStages;
-        const uint32_t use = static_cast<uint32_t>(it / kStages);
-        if (it >= kStages && !mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err)) break;
-        const int32_t kc = it * kBK;  // contraction offset
-        const uint32_t a_dst = smem_u32(sA + s * kAStageBytes);
-        if (MODE == MODE_SGRAD) {
-          mbar_arrive_expect_tx(&afull[s], kAStageBytes + kBStageBytes);
-          const uint32_t b_dst = smem_u32(sB + s * kBStageBytes);
-          // dY^T tile: two 64(n) x 64(m) boxes; X tile: four 64(k) x 64(m) boxes.
-          for (int j = 0; j < kBM / 64; ++j)
-            tma_load_2d(a_dst + j * (kBK * 128), &tmA, &afull[s], static_cast<int32_t>(row0) + 64 * j, kc);
-          for (int j = 0; j < kBN / 64; ++j)
-            tma_load_2d(b_dst + j * (kBK * 128), &tmB, &afull[s], static_cast<int32_t>(col0) + 64 * j, kc);
-        } else {
-          mbar_arrive_expect_tx(&afull[s], kAStageBytes);
-          tma_load_2d(a_dst, &tmA, &afull[s], kc, static_cast<int32_t>(row0));
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        int tm, tn;
+        tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+        const int32_t row0 = tm * kBM, col0 = tn * kBN;
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t use = static_cast<uint32_t>(it / kStages);
+          if (it >= kStages && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          mbar_arrive_expect_tx(&afull[s], C::kTxBytes);
+          const uint32_t a_dst = smem_u32(stage_a(s));
+          const int32_t kc = kb * kBK;
+          if (MODE == MODE_SGRAD) {
+            const uint32_t b_dst = smem_u32(stage_b(s));
+            // dY^T tile: two 64(n) x 64(m) boxes; X tile: four 64(k) x 64(m) boxes (MN-major).
+            for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * (kBK * 128), &tmA, &afull[s], row0 + 64 * j, kc);
+            for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * (kBK * 128), &tmB, &afull[s], col0 + 64 * j, kc);
+          } else {
+            const uint32_t c_dst = smem_u32(stage_c(s));
+            tma_load_2d(a_dst, &tmA, &afull[s], kc, row0);
+            if (MODE == MODE_FWD)  // codes [N, K/2]: 256 rows x 32 bytes at (byte k/2, row n)
+              tma_load_2d(c_dst, &tmB, &afull[s], kc / 2, col0);
+            else                   // 64 rows x 128 bytes, 128-byte swizzle
+              tma_load_2d(c_dst, &tmB, &afull[s], col0 / 2, kc);
+          }
         }
-        issued = it + 1;
       }
       if (*abort_flag) {
         // Let every issued copy land before the CTA's shared memory goes away.
-        for (int it = (issued > kStages ? issued - kStages : 0); it < issued; ++it)
-          mbar_drain(&afull[it % kStages], static_cast<uint32_t>(it / kStages) & 1u);
+        for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+          mbar_drain(&afull[i % kStages], static_cast<uint32_t>(i / kStages) & 1u);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, kBN, MODE == MODE_SGRAD ? 1 : 0, MODE == MODE_FWD ? 0 : 1);
+      int it = 0, tc = 0;
       bool ok = true;
-      for (int it = 0; it < num_k && ok; ++it) {
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tc) {
+        const int ab = tc & 1;
+        const uint32_t au = static_cast<uint32_t>(tc >> 1);
+        if (tc >= 2 && !(ok = mbar_wait(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + ab * kTmemCols;
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
+          ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
+          if (ok && C::kDecode) ok = mbar_wait(&bfull[s], ph, abort_flag, p.err);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(stage_a(s));
+          const uint32_t b_base = smem_u32(stage_b(s));
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = MODE == MODE_SGRAD ? smem_desc_sw128(a_base + kk * 2048, kBK * 128, 1024)
+                                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+            const uint64_t bd = MODE == MODE_FWD ? smem_desc_sw128(b_base + kk * 32, 16, 1024)
+                                                 : smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
+            umma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (ok) umma_commit(&tfull[ab]);
+      }
+      umma_commit(drain);  // completes once every MMA issued above has finished
+      mbar_drain(drain, 0);
+    }
+  } else if (warp >= C::kEpiWarps) {
+    // ------------------------------------------------------ decode (FWD / DX)
+    if (C::kDecode) {
+      const int dt = threadIdx.x - 32 * C::kEpiWarps;  // 0..255, two units per k-step
+      int it = 0;
+      bool ok = true;
+      // scale bytes are prefetched one k-step ahead (codes arrive by TMA)
+      int tile = blockIdx.x, kb = 0;
+      int tm = 0, tn = 0;
+      if (tile < total) tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+      uint32_t sc[2] = {0u, 0u};
+      if (tile < total)
+        for (int i = 0; i < 2; ++i) {
+          int64_t n, k;
+          unit_coords<MODE>(dt + 256 * i, static_cast<int64_t>(tn) * kBN, 0, n, k);
+          sc[i] = load_unit_scale<FMT>(p, n, k);
+        }
+      while (tile < total && ok) {
+        // next position in the flattened (tile, k-step) walk
+        int ntile = tile, nkb = kb + 1, ntm = tm, ntn = tn;
+        if (nkb == num_k) {
+          nkb = 0;
+          ntile += gridDim.x;
+          if (ntile < total) tile_coords(ntile, p.tiles_m, p.tiles_n, ntm, ntn);
+        }
+        uint32_t nsc[2] = {0u, 0u};
+        if (ntile < total)
+          for (int i = 0; i < 2; ++i) {
+            int64_t n, k;
+            unit_coords<MODE>(dt + 256 * i, static_cast<int64_t>(ntn) * kBN, nkb, n, k);
+            nsc[i] = load_unit_scale<FMT>(p, n, k);
+          }
         const int s = it % kStages;
         const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-        ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
-        if (ok && MODE != MODE_SGRAD) ok = mbar_wait(&bfull[s], ph, abort_flag, p.err);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t a_base = smem_u32(sA + s * kAStageBytes);
-        const uint32_t b_base = smem_u32(sB + s * kBStageBytes);
+        if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
+        const uint32_t b_base = smem_u32(stage_b(s));
+        const uint32_t c_base = smem_u32(stage_c(s));
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          uint64_t ad, bd;
-          if (MODE == MODE_SGRAD) {
-            ad = smem_desc_sw128(a_base + kk * 2048, kBK * 128, 1024);
-          } else {
-            ad = smem_desc_sw128(a_base + kk * 32, 16, 1024);
-          }
-          if (MODE == MODE_FWD) {
-            bd = smem_desc_sw128(b_base + kk * 32, 16, 1024);
-          } else {
-            bd = smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
-          }
-          umma_bf16(tmem_base, ad, bd, idesc, (it > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&empty[s]);
-      }
-      if (ok) {
-        umma_commit(tfull);
-      } else {
-        umma_commit(drain);  // completes once every MMA issued so far has finished
-        mbar_drain(drain, 0);
-      }
-    }
-  } else {
-    // ------------------------------------------------------ decode (warps 0-3)
-    if (MODE != MODE_SGRAD) {
-      const int t = threadIdx.x;  // 0..127
-      const int64_t K2 = p.K / 2;
-      const int64_t G = p.K / B;
-      // 512 units of 32 consecutive weight elements per stage, 4 per thread.
-      uint4 cw[4], cn[4];
-      uint32_t sw[4], sn[4];
-      auto load_units = [&](int it, uint4 (&c)[4], uint32_t (&sc)[4]) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int u = t + 128 * i;
-          int64_t n, k;
-          if (MODE == MODE_FWD) {  // tile rows = out features n, cols = k (K-major)
-            n = col0 + (u >> 1);
-            k = static_cast<int64_t>(it) * kBK + 32 * (u & 1);
-          } else {  // tile rows = contraction n (MN-major), cols = 256 k-values
-            const int j = (u & 7) + 8 * (u >> 6);
-            const int part = (u >> 3) & 7;
-            n = static_cast<int64_t>(it) * kBK + j;
-            k = col0 + 32 * part;
-          }
-          if (n < p.N && k < p.K) {
-            c[i] = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * K2 + k / 2));
-            if (FMT == 0)
-              sc[i] = __ldg(reinterpret_cast<const unsigned short *>(p.scales + n * G + k / 16));
-            else
-              sc[i] = __ldg(p.scales + n * G + k / 32);
-          } else {
-            c[i] = make_uint4(0u, 0u, 0u, 0u);
-            sc[i] = FMT == 0 ? 0x3838u : 127u;  // any finite scale; the codes are zero
-          }
-        }
-      };
-      if (num_k > 0) load_units(0, cw, sw);
-      for (int it = 0; it < num_k; ++it) {
-        const int s = it % kStages;
-        const uint32_t use = static_cast<uint32_t>(it / kStages);
-        if (it + 1 < num_k) load_units(it + 1, cn, sn);
-        if (it >= kStages && !mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err)) break;
-        const uint32_t b_base = smem_u32(sB + s * kBStageBytes);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int u = t + 128 * i;
+        for (int i = 0; i < 2; ++i) {
+          const int u = dt + 256 * i;
           uint32_t sc_lo, sc_hi;
           if (FMT == 0) {
-            sc_lo = scale_bf16x2<0>(sw[i] & 0xFFu);
-            sc_hi = scale_bf16x2<0>(sw[i] >> 8);
+            sc_lo = scale_bf16x2<0>(sc[i] & 0xFFu);
+            sc_hi = scale_bf16x2<0>(sc[i] >> 8);
           } else {
-            sc_lo = sc_hi = scale_bf16x2<1>(sw[i]);
+            sc_lo = sc_hi = scale_bf16x2<1>(sc[i]);
           }
-          const uint32_t words[4] = {cw[i].x, cw[i].y, cw[i].z, cw[i].w};
+          uint4 cw;
+          if (MODE == MODE_FWD) {
+            cw = lds128(c_base + (u >> 1) * 32 + (u & 1) * 16);
+          } else {
+            const int j = (u & 7) + 8 * (u >> 6);
+            const int part = (u >> 3) & 7;
+            cw = lds128(c_base + j * 128 + ((part ^ (j & 7)) << 4));
+          }
+          const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             uint32_t o[4];
             e2m1x8_to_bf16(words[c], o);
-            const uint32_t sc = c < 2 ? sc_lo : sc_hi;
+            const uint32_t scv = c < 2 ? sc_lo : sc_hi;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], sc);
+            for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
             uint32_t addr;
             if (MODE == MODE_FWD) {
               const int r = u >> 1;
@@ -456,9 +529,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
               const int j = (u & 7) + 8 * (u >> 6);
               const int part = (u >> 3) & 7;
-              const int atom = part >> 1;
               const int chunk = 4 * (part & 1) + c;
-              addr = b_base + atom * (kBK * 128) + j * 128 + ((chunk ^ (j & 7)) << 4);
+              addr = b_base + (part >> 1) * (kBK * 128) + j * 128 + ((chunk ^ (j & 7)) << 4);
             }
             st_shared_v4(addr, o[0], o[1], o[2], o[3]);
           }
@@ -466,109 +538,132 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bfull[s]);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          cw[i] = cn[i];
-          sw[i] = sn[i];
-        }
+        ++it;
+        tile = ntile;
+        kb = nkb;
+        tm = ntm;
+        tn = ntn;
+        sc[0] = nsc[0];
+        sc[1] = nsc[1];
       }
     }
-
+  } else {
     // ------------------------------------------------------ epilogue (warps 0-3)
-    const bool ok = num_k > 0 && mbar_wait(tfull, 0, abort_flag, p.err);
-    tc_fence_after();
     const int r = warp * 32 + lane;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
-    if (MODE != MODE_SGRAD) {
-      const int64_t grow = row0 + r;
-      const float scale = FMT == 0 ? p.ws2 : 1.0f;
-      __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(t_row + c0, v);
-        tmem_ld_wait();
-        if (!ok || grow >= Mg) continue;
+    int tc = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++tc) {
+      int tm, tn;
+      tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+      const int64_t row0 = static_cast<int64_t>(tm) * kBM, col0 = static_cast<int64_t>(tn) * kBN;
+      const int ab = tc & 1;
+      const uint32_t au = static_cast<uint32_t>(tc >> 1);
+      if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
+      tc_fence_after();
+      const uint32_t t_buf = t_row + ab * kTmemCols;
+      if (MODE != MODE_SGRAD) {
+        const int64_t Mg = p.M;
+        const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
+        const int64_t grow = row0 + r;
+        const float scale = FMT == 0 ? p.ws2 : 1.0f;
+        __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
+        for (int c0 = 0; c0 < kBN; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld32(t_buf + c0, v);
+          tmem_ld_wait();
+          if (grow >= Mg) continue;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int64_t gc = col0 + c0 + 8 * q;
-          if (gc >= Ng) continue;
-          uint32_t packed[4];
+          for (int q = 0; q < 4; ++q) {
+            const int64_t gc = col0 + c0 + 8 * q;
+            if (gc >= Ng) continue;
+            uint32_t packed[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float a = __uint_as_float(v[8 * q + 2 * e]) * scale;
-            const float b = __uint_as_float(v[8 * q + 2 * e + 1]) * scale;
-            const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-            packed[e] = *reinterpret_cast<const uint32_t *>(&h);
+            for (int e = 0; e < 4; ++e) {
+              const float a = __uint_as_float(v[8 * q + 2 * e]) * scale;
+              const float b = __uint_as_float(v[8 * q + 2 * e + 1]) * scale;
+              const __nv_bfloat162 h2 = __floats2bfloat162_rn(a, b);
+              packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
+            }
+            *reinterpret_cast<uint4 *>(out + grow * Ng + gc) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
           }
-          *reinterpret_cast<uint4 *>(out + grow * Ng + gc) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        }
+      } else {
+        constexpr int B = FMT == 0 ? 16 : 32;
+        const int64_t n = row0 + r;
+        const int64_t G = p.K / B;
+        float *g = static_cast<float *>(p.out);
+        for (int c0 = 0; c0 < kBN; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld32(t_buf + c0, v);
+          tmem_ld_wait();
+          const int64_t k = col0 + c0;
+          if (n >= p.N || k >= p.K) continue;
+          const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
+          const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+          float part[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            uint32_t o[4];
+            e2m1x8_to_bf16(words[c], o);
+            float acc = 0.f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
+              acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
+            }
+            part[c] = acc;
+          }
+          if (FMT == 0) {
+            const int64_t b = k / 16;
+            float g0 = part[0] + part[1];
+            float g1 = part[2] + part[3];
+            if (p.mask) {
+              g0 *= static_cast<float>(p.mask[n * G + b]);
+              g1 *= static_cast<float>(p.mask[n * G + b + 1]);
+            }
+            *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
+          } else {
+            const int64_t b = k / 32;
+            float g0 = (part[0] + part[1]) + (part[2] + part[3]);
+            if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
+            g[n * G + b] = g0;
+          }
         }
       }
-    } else {
-      const int64_t n = row0 + r;
-      const int64_t G = p.K / B;
-      float *g = static_cast<float *>(p.out);
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(t_row + c0, v);
-        tmem_ld_wait();
-        const int64_t k = col0 + c0;
-        if (!ok || n >= p.N || k >= p.K) continue;
-        const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
-        const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
-        float part[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint32_t o[4];
-          e2m1x8_to_bf16(words[c], o);
-          float acc = 0.f;
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
-            acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
-          }
-          part[c] = acc;
-        }
-        if (FMT == 0) {
-          const int64_t b = k / 16;
-          float g0 = part[0] + part[1];
-          float g1 = part[2] + part[3];
-          if (p.mask) {
-            g0 *= static_cast<float>(p.mask[n * G + b]);
-            g1 *= static_cast<float>(p.mask[n * G + b + 1]);
-          }
-          *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
-        } else {
-          const int64_t b = k / 32;
-          float g0 = (part[0] + part[1]) + (part[2] + part[3]);
-          if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
-          g[n * G + b] = g0;
-        }
-      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[ab]);
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == C::kMmaWarp) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc(tmem_base, 2 * kTmemCols);
   }
 }
 
 template <int MODE, int FMT>
-cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, cudaStream_t stream) {
-  static bool attr_done = false;  // per process; the attribute is per function
-  if (!attr_done) {
+cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
+                       cudaStream_t stream) {
+  using C = Cfg<MODE>;
+  static int attr_done_mask = 0;  // per device ordinal (first 31)
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (!(attr_done_mask & (1 << (dev & 31)))) {
     cudaError_t e = cudaFuncSetAttribute(sq_gemm_kernel<MODE, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kSmemBytes);
+                                         C::kSmemBytes);
     if (e != cudaSuccess) return e;
-    attr_done = true;
+    attr_done_mask |= 1 << (dev & 31);
   }
   const int64_t Mg = MODE == MODE_SGRAD ? a.N : a.M;
   const int64_t Ng = MODE == MODE_FWD ? a.N : a.K;
-  dim3 grid(static_cast<unsigned>((Mg + kBM - 1) / kBM), static_cast<unsigned>((Ng + kBN - 1) / kBN));
-  KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err};
-  sq_gemm_kernel<MODE, FMT><<<grid, kThreads, kSmemBytes, stream>>>(tmA, tmB, p);
+  KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err,
+            static_cast<int>((Mg + kBM - 1) / kBM), static_cast<int>((Ng + kBN - 1) / kBN)};
+  const int64_t total = static_cast<int64_t>(p.tiles_m) * p.tiles_n;
+  const int grid = static_cast<int>(total < sm_count ? total : sm_count);
+  sq_gemm_kernel<MODE, FMT><<<grid, C::kThreads, C::kSmemBytes, stream>>>(tmA, tmB, p);
   return cudaGetLastError();
 }
 
@@ -576,15 +671,14 @@ cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensor
 
 cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
                         cudaStream_t stream) {
-  (void)sm_count;
   if (a.fmt == 0) {
-    if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 0>(a, tmA, tmB, stream);
-    if (a.mode == MODE_DX) return launch_one<MODE_DX, 0>(a, tmA, tmB, stream);
-    return launch_one<MODE_SGRAD, 0>(a, tmA, tmB, stream);
+    if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 0>(a, tmA, tmB, sm_count, stream);
+    if (a.mode == MODE_DX) return launch_one<MODE_DX, 0>(a, tmA, tmB, sm_count, stream);
+    return launch_one<MODE_SGRAD, 0>(a, tmA, tmB, sm_count, stream);
   }
-  if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 1>(a, tmA, tmB, stream);
-  if (a.mode == MODE_DX) return launch_one<MODE_DX, 1>(a, tmA, tmB, stream);
-  return launch_one<MODE_SGRAD, 1>(a, tmA, tmB, stream);
+  if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 1>(a, tmA, tmB, sm_count, stream);
+  if (a.mode == MODE_DX) return launch_one<MODE_DX, 1>(a, tmA, tmB, sm_count, stream);
+  return launch_one<MODE_SGRAD, 1>(a, tmA, tmB, sm_count, stream);
 }
 
 }  // namespace sqi
