@@ -275,11 +275,17 @@ struct KParams {
   int tiles_m, tiles_n;
 };
 
+#ifndef SQ_DECODE_WARPS
+#define SQ_DECODE_WARPS 16
+#endif
+static_assert(512 % (32 * SQ_DECODE_WARPS) == 0, "decode warps must divide the 512 units of a k-step");
+
 template <int MODE>
 struct Cfg {
   static constexpr bool kDecode = MODE != MODE_SGRAD;
   static constexpr int kEpiWarps = 4;                      // warps 0-3: TMEM lanes 0-127
-  static constexpr int kDecWarps = kDecode ? 8 : 0;        // warps 4-11
+  static constexpr int kDecWarps = kDecode ? SQ_DECODE_WARPS : 0;  // warps 4 .. 3 + kDecWarps
+  static constexpr int kUnits = kDecode ? 512 / (32 * (kDecode ? kDecWarps : 1)) : 1;  // 32-weight units per thread per k-step
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
   static constexpr int kMmaWarp = kTmaWarp + 1;
   static constexpr int kThreads = 32 * (kMmaWarp + 1);
@@ -294,6 +300,7 @@ struct Cfg {
 // column index varying slowest inside a group, so the CTAs resident at any
 // moment share a few row panels and column panels in L2.
 constexpr int kGroup = 8;
+
 
 __device__ __forceinline__ void tile_coords(int id, int tiles_m, int tiles_n, int &tm, int &tn) {
   const int per_group = kGroup * tiles_n;
@@ -461,20 +468,22 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   } else if (warp >= C::kEpiWarps) {
     // ------------------------------------------------------ decode (FWD / DX)
     if (C::kDecode) {
-      const int dt = threadIdx.x - 32 * C::kEpiWarps;  // 0..255, two units per k-step
+      constexpr int kDecThreads = 32 * C::kDecWarps;
+      constexpr int kU = C::kUnits;
+      const int dt = threadIdx.x - 32 * C::kEpiWarps;  // this thread owns units dt + kDecThreads * i
       int it = 0;
       bool ok = true;
       // scale bytes are prefetched one k-step ahead (codes arrive by TMA)
       int tile = blockIdx.x, kb = 0;
       int tm = 0, tn = 0;
       if (tile < total) tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-      uint32_t sc[2] = {0u, 0u};
-      if (tile < total)
-        for (int i = 0; i < 2; ++i) {
-          int64_t n, k;
-          unit_coords<MODE>(dt + 256 * i, static_cast<int64_t>(tn) * kBN, 0, n, k);
-          sc[i] = load_unit_scale<FMT>(p, n, k);
-        }
+      uint32_t sc[kU];
+#pragma unroll
+      for (int i = 0; i < kU; ++i) {
+        int64_t n, k;
+        unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(tn) * kBN, 0, n, k);
+        sc[i] = tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
+      }
       while (tile < total && ok) {
         // next position in the flattened (tile, k-step) walk
         int ntile = tile, nkb = kb + 1, ntm = tm, ntn = tn;
@@ -483,21 +492,25 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           ntile += gridDim.x;
           if (ntile < total) tile_coords(ntile, p.tiles_m, p.tiles_n, ntm, ntn);
         }
-        uint32_t nsc[2] = {0u, 0u};
-        if (ntile < total)
-          for (int i = 0; i < 2; ++i) {
-            int64_t n, k;
-            unit_coords<MODE>(dt + 256 * i, static_cast<int64_t>(ntn) * kBN, nkb, n, k);
-            nsc[i] = load_unit_scale<FMT>(p, n, k);
-          }
+        uint32_t nsc[kU];
+#pragma unroll
+        for (int i = 0; i < kU; ++i) {
+          int64_t n, k;
+          unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(ntn) * kBN, nkb, n, k);
+          nsc[i] = ntile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
+        }
         const int s = it % kStages;
         const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-        if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
+        // one lane polls the barrier (32 polling lanes serialise), the warp follows
+        if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
+        ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+        __syncwarp();
+        if (!ok) break;
         const uint32_t b_base = smem_u32(stage_b(s));
         const uint32_t c_base = smem_u32(stage_c(s));
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const int u = dt + 256 * i;
+        for (int i = 0; i < kU; ++i) {
+          const int u = dt + kDecThreads * i;
           uint32_t sc_lo, sc_hi;
           if (FMT == 0) {
             sc_lo = scale_bf16x2<0>(sc[i] & 0xFFu);
@@ -543,8 +556,8 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         kb = nkb;
         tm = ntm;
         tn = ntn;
-        sc[0] = nsc[0];
-        sc[1] = nsc[1];
+#pragma unroll
+        for (int i = 0; i < kU; ++i) sc[i] = nsc[i];
       }
     }
   } else {
