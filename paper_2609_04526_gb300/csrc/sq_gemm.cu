@@ -104,6 +104,35 @@ __device__ __noinline__ void mbar_drain(uint64_t *bar, uint32_t parity) {
     if (globaltimer() - t0 > kWaitLimitNs) return;
 }
 
+// The same bounded wait with cluster-scope acquire, for barriers that threads of
+// the peer CTA arrive on with cluster-scope release.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __noinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, volatile int *abort_flag, int *err) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  while (true) {
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      atomicOr(err, kErrWaitTimeout);
+      return false;
+    }
+  }
+}
+
 __device__ __forceinline__ void fence_barrier_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
@@ -279,6 +308,12 @@ struct KParams {
 #define SQ_DECODE_WARPS 16
 #endif
 static_assert(512 % (32 * SQ_DECODE_WARPS) == 0, "decode warps must divide the 512 units of a k-step");
+#ifndef SQ_PAIR_DEC_GROUPS
+#define SQ_PAIR_DEC_GROUPS 2
+#endif
+#ifndef SQ_SCALE_DEPTH
+#define SQ_SCALE_DEPTH 4
+#endif
 
 template <int MODE>
 struct Cfg {
@@ -470,94 +505,99 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     if (C::kDecode) {
       constexpr int kDecThreads = 32 * C::kDecWarps;
       constexpr int kU = C::kUnits;
+      constexpr int kD = SQ_SCALE_DEPTH;  // scale bytes are loaded kD k-steps ahead (codes arrive by TMA)
       const int dt = threadIdx.x - 32 * C::kEpiWarps;  // this thread owns units dt + kDecThreads * i
-      int it = 0;
-      bool ok = true;
-      // scale bytes are prefetched one k-step ahead (codes arrive by TMA)
-      int tile = blockIdx.x, kb = 0;
-      int tm = 0, tn = 0;
-      if (tile < total) tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-      uint32_t sc[kU];
-#pragma unroll
-      for (int i = 0; i < kU; ++i) {
-        int64_t n, k;
-        unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(tn) * kBN, 0, n, k);
-        sc[i] = tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
-      }
-      while (tile < total && ok) {
-        // next position in the flattened (tile, k-step) walk
-        int ntile = tile, nkb = kb + 1, ntm = tm, ntn = tn;
-        if (nkb == num_k) {
-          nkb = 0;
-          ntile += gridDim.x;
-          if (ntile < total) tile_coords(ntile, p.tiles_m, p.tiles_n, ntm, ntn);
+      // position in the flattened (tile, k-step) walk: current and kD steps ahead
+      int c_tile = blockIdx.x, c_kb = 0, c_tn = 0, c_tm = 0;
+      if (c_tile < total) tile_coords(c_tile, p.tiles_m, p.tiles_n, c_tm, c_tn);
+      int a_tile = c_tile, a_kb = 0, a_tn = c_tn, a_tm = c_tm;
+      auto advance = [&](int &tile, int &kb, int &tm, int &tn) {
+        if (++kb == num_k) {
+          kb = 0;
+          tile += gridDim.x;
+          if (tile < total) tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
         }
-        uint32_t nsc[kU];
+      };
+      uint32_t sc[kD][kU];
+#pragma unroll
+      for (int d = 0; d < kD; ++d) {
 #pragma unroll
         for (int i = 0; i < kU; ++i) {
           int64_t n, k;
-          unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(ntn) * kBN, nkb, n, k);
-          nsc[i] = ntile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
+          unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(a_tn) * kBN, a_kb, n, k);
+          sc[d][i] = a_tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
         }
-        const int s = it % kStages;
-        const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-        // one lane polls the barrier (32 polling lanes serialise), the warp follows
-        if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
-        ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
-        __syncwarp();
-        if (!ok) break;
-        const uint32_t b_base = smem_u32(stage_b(s));
-        const uint32_t c_base = smem_u32(stage_c(s));
+        advance(a_tile, a_kb, a_tm, a_tn);
+      }
+      int it = 0;
+      bool ok = true;
+      while (c_tile < total && ok) {
 #pragma unroll
-        for (int i = 0; i < kU; ++i) {
-          const int u = dt + kDecThreads * i;
-          uint32_t sc_lo, sc_hi;
-          if (FMT == 0) {
-            sc_lo = scale_bf16x2<0>(sc[i] & 0xFFu);
-            sc_hi = scale_bf16x2<0>(sc[i] >> 8);
-          } else {
-            sc_lo = sc_hi = scale_bf16x2<1>(sc[i]);
-          }
-          uint4 cw;
-          if (MODE == MODE_FWD) {
-            cw = lds128(c_base + (u >> 1) * 32 + (u & 1) * 16);
-          } else {
-            const int j = (u & 7) + 8 * (u >> 6);
-            const int part = (u >> 3) & 7;
-            cw = lds128(c_base + j * 128 + ((part ^ (j & 7)) << 4));
-          }
-          const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+        for (int d = 0; d < kD; ++d) {
+          if (c_tile >= total || !ok) break;
+          const int s = it % kStages;
+          const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
+          // one lane polls the barrier (32 polling lanes serialise), the warp follows
+          if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
+          ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+          __syncwarp();
+          if (!ok) break;
+          const uint32_t b_base = smem_u32(stage_b(s));
+          const uint32_t c_base = smem_u32(stage_c(s));
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            uint32_t o[4];
-            e2m1x8_to_bf16(words[c], o);
-            const uint32_t scv = c < 2 ? sc_lo : sc_hi;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
-            uint32_t addr;
+          for (int i = 0; i < kU; ++i) {
+            const int u = dt + kDecThreads * i;
+            uint32_t sc_lo, sc_hi;
+            if (FMT == 0) {
+              sc_lo = scale_bf16x2<0>(sc[d][i] & 0xFFu);
+              sc_hi = scale_bf16x2<0>(sc[d][i] >> 8);
+            } else {
+              sc_lo = sc_hi = scale_bf16x2<1>(sc[d][i]);
+            }
+            uint4 cw;
             if (MODE == MODE_FWD) {
-              const int r = u >> 1;
-              const int chunk = 4 * (u & 1) + c;
-              addr = b_base + (r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4);
+              cw = lds128(c_base + (u >> 1) * 32 + (u & 1) * 16);
             } else {
               const int j = (u & 7) + 8 * (u >> 6);
               const int part = (u >> 3) & 7;
-              const int chunk = 4 * (part & 1) + c;
-              addr = b_base + (part >> 1) * (kBK * 128) + j * 128 + ((chunk ^ (j & 7)) << 4);
+              cw = lds128(c_base + j * 128 + ((part ^ (j & 7)) << 4));
             }
-            st_shared_v4(addr, o[0], o[1], o[2], o[3]);
-          }
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bfull[s]);
-        ++it;
-        tile = ntile;
-        kb = nkb;
-        tm = ntm;
-        tn = ntn;
+            const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
-        for (int i = 0; i < kU; ++i) sc[i] = nsc[i];
+            for (int c = 0; c < 4; ++c) {
+              uint32_t o[4];
+              e2m1x8_to_bf16(words[c], o);
+              const uint32_t scv = c < 2 ? sc_lo : sc_hi;
+#pragma unroll
+              for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
+              uint32_t addr;
+              if (MODE == MODE_FWD) {
+                const int r = u >> 1;
+                const int chunk = 4 * (u & 1) + c;
+                addr = b_base + (r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4);
+              } else {
+                const int j = (u & 7) + 8 * (u >> 6);
+                const int part = (u >> 3) & 7;
+                const int chunk = 4 * (part & 1) + c;
+                addr = b_base + (part >> 1) * (kBK * 128) + j * 128 + ((chunk ^ (j & 7)) << 4);
+              }
+              st_shared_v4(addr, o[0], o[1], o[2], o[3]);
+            }
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bfull[s]);
+          // refill this ring slot with the scales of the position kD steps ahead
+#pragma unroll
+          for (int i = 0; i < kU; ++i) {
+            int64_t n, k;
+            unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(a_tn) * kBN, a_kb, n, k);
+            sc[d][i] = a_tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
+          }
+          advance(a_tile, a_kb, a_tm, a_tn);
+          advance(c_tile, c_kb, c_tm, c_tn);
+          ++it;
+        }
       }
     }
   } else {
@@ -657,6 +697,417 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   }
 }
 
+// ------------------------------------------------------------- CTA-pair kernel (FWD / DX)
+//
+// Two CTAs of a cluster share one 256 x 256 output tile through
+// tcgen05.mma.cta_group::2 (M = 256, N = 256): each CTA holds its 128-row half
+// of the activation tile (A) and decodes its 128-row (FWD) or 128-column (DX)
+// half of the weight tile (B), so every SM decodes half as many weights per MMA
+// cycle as in the single-CTA kernel. The leader CTA (cluster rank 0) issues the
+// MMAs; its stage barriers collect the decode warps of both CTAs, and each MMA
+// commit is multicast to the stage / accumulator barriers of both CTAs. Each CTA
+// keeps its 128 accumulator rows in its own TMEM and runs its own epilogue.
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Shared-memory address of the same variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+
+// TMEM allocation for a CTA pair: one warp of each CTA executes these collectively.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on `bar` in both CTAs of the pair when the pair's MMAs issued so far complete.
+__device__ __forceinline__ void umma_commit_pair_mc(uint64_t *bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(static_cast<unsigned short>(3))
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit_pair(uint64_t *bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+struct PairCfg {
+  static constexpr int kEpiWarps = 4;    // warps 0-3
+  static constexpr int kDecGroups = SQ_PAIR_DEC_GROUPS;  // decode groups take k-steps in turn
+  static constexpr int kDecWarps = 8 * kDecGroups;       // 8 warps per group: one 32-weight unit per thread
+  static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
+  static constexpr int kMmaWarp = kTmaWarp + 1;
+  static constexpr int kSigWarp0 = kMmaWarp + 1;
+  static constexpr int kSigWarps = 4;    // peer CTA: forward "half decoded" to the leader, k-steps in turn
+  static constexpr int kThreads = 32 * (kSigWarp0 + kSigWarps);
+  static constexpr int kStages = 6;
+  static constexpr int kA = 128 * kBK * 2;  // 16 KiB: this CTA's 128 activation rows
+  static constexpr int kB = 128 * kBK * 2;  // 16 KiB: this CTA's half of the decoded weight tile
+  static constexpr int kC = 4096;           // packed codes of that half
+  static constexpr int kStageBytes = kA + kB + kC;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 512;
+  static constexpr uint32_t kTx = kA + kC;
+  static constexpr int kTile = 256;         // output tile is kTile x kTile per pair
+};
+
+// Weight coordinates of decode unit u (0..255) of this CTA's half at k-step kb.
+template <int MODE>
+__device__ __forceinline__ void pair_unit_coords(int u, int64_t half0, int kb, int64_t &n, int64_t &k) {
+  if (MODE == MODE_FWD) {  // 128 out-feature rows x 64 k
+    n = half0 + (u >> 1);
+    k = static_cast<int64_t>(kb) * kBK + 32 * (u & 1);
+  } else {  // 64 contraction rows x 128 k-columns
+    n = static_cast<int64_t>(kb) * kBK + (u & 7) + 8 * (u >> 5);
+    k = half0 + 32 * ((u >> 3) & 3);
+  }
+}
+
+template <int MODE, int FMT>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1)
+    sq_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmC,
+                        const KParams p) {
+  using C = PairCfg;
+  constexpr int S = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + S * C::kStageBytes);
+  uint64_t *afull = bars;             // this CTA's TMA tiles landed            (1 arrival + tx)
+  uint64_t *bready = bars + S;        // this CTA's weight half decoded          (8 decode-warp arrivals)
+  uint64_t *empty = bars + 2 * S;     // pair MMAs reading the stage completed   (multicast commit)
+  uint64_t *pready = bars + 3 * S;    // leader: the peer's half decoded         (1 cluster arrival)
+  uint64_t *tfull = bars + 4 * S;     // [2] accumulator buffer complete         (multicast commit)
+  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained      (2 x kEpiWarps arrivals)
+  uint64_t *drain = tempty + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int cluster = blockIdx.x >> 1;
+  const int nclusters = gridDim.x >> 1;
+  const int total = p.tiles_m * p.tiles_n;
+  const int64_t Kg = MODE == MODE_FWD ? p.K : p.N;
+  const int num_k = static_cast<int>((Kg + kBK - 1) / kBK);
+
+  auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
+  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
+  auto stage_c = [&](int s) { return smem + s * C::kStageBytes + C::kA + C::kB; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&afull[s], 1);
+      mbar_init(&bready[s], 8);  // one arrival per decode warp of the group that owns the k-step
+      mbar_init(&empty[s], 1);
+      mbar_init(&pready[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 2 * C::kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == C::kMmaWarp) tmem_alloc_pair(tmem_slot, 2 * kTmemCols);
+  if (warp == C::kTmaWarp && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmC);
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == C::kTmaWarp) {
+    // ------------------------------------------------------ TMA producer (both CTAs)
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        int tm, tn;
+        tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+        const int32_t row0 = tm * C::kTile + 128 * static_cast<int32_t>(rank);
+        const int32_t half0 = tn * C::kTile + 128 * static_cast<int32_t>(rank);
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % S;
+          const uint32_t use = static_cast<uint32_t>(it / S);
+          if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          mbar_arrive_expect_tx(&afull[s], C::kTx);
+          tma_load_2d(smem_u32(stage_a(s)), &tmA, &afull[s], kb * kBK, row0);
+          if (MODE == MODE_FWD)  // codes: 128 rows x 32 bytes
+            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], kb * (kBK / 2), half0);
+          else                   // codes: 64 rows x 64 bytes, 64-byte swizzle
+            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], half0 / 2, kb * kBK);
+        }
+      }
+      if (*abort_flag) {
+        for (int i = (it > S ? it - S : 0); i < it; ++i)
+          mbar_drain(&afull[i % S], static_cast<uint32_t>(i / S) & 1u);
+      }
+    }
+  } else if (warp == C::kMmaWarp) {
+    // ------------------------------------------------------ MMA issuer (leader CTA)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
+      int it = 0, tc = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
+        const int ab = tc & 1;
+        const uint32_t au = static_cast<uint32_t>(tc >> 1);
+        if (tc >= 2 && !(ok = mbar_wait_cluster(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + ab * kTmemCols;
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % S;
+          const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+          ok = mbar_wait(&bready[s], ph, abort_flag, p.err);                // own half
+          if (ok) ok = mbar_wait_cluster(&pready[s], ph, abort_flag, p.err);  // the peer's half
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(stage_a(s));
+          const uint32_t b_base = smem_u32(stage_b(s));
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = smem_desc_sw128(a_base + kk * 32, 16, 1024);
+            const uint64_t bd = MODE == MODE_FWD ? smem_desc_sw128(b_base + kk * 32, 16, 1024)
+                                                 : smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
+            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit_pair_mc(&empty[s]);
+        }
+        if (ok) umma_commit_pair_mc(&tfull[ab]);
+      }
+      umma_commit_pair(drain);
+      mbar_drain(drain, 0);
+    }
+  } else if (warp >= C::kSigWarp0) {
+    // ------------------------------------------------------ signal warps (peer CTA)
+    // Forward "this CTA's weight half of stage s is decoded" to the leader with
+    // one cluster-scope release per k-step. A cluster-scope release holds the
+    // issuing warp for a long time, so it is kept off the decode warps and the
+    // k-steps are spread over kSigWarps warps.
+    if (rank == 1 && lane == 0) {
+      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
+      const int iters = my_tiles * num_k;
+      const uint32_t leader_pready = mapa_shared(smem_u32(&pready[0]), 0);
+      for (int it = warp - C::kSigWarp0; it < iters; it += C::kSigWarps) {
+        const int s = it % S;
+        if (!mbar_wait(&bready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
+        mbar_arrive_cluster(leader_pready + 8u * s);
+      }
+    }
+  } else if (warp >= C::kEpiWarps) {
+    // ------------------------------------------------------ decode (both CTAs)
+    // Group g of 8 warps decodes the k-steps it = g, g + kDecGroups, ... of the
+    // flattened (tile, k-step) walk; every thread owns one 32-weight unit.
+    constexpr int kD = SQ_SCALE_DEPTH;
+    constexpr int kG = C::kDecGroups;
+    const int dw = warp - C::kEpiWarps;
+    const int group = dw / 8;
+    const int u = (dw % 8) * 32 + lane;  // this thread's unit, 0..255
+    // walker over the flattened walk: position -> (tile, k-step)
+    struct Pos {
+      int tile, kb, tm, tn;
+    };
+    auto step_by = [&](Pos &q, int n) {
+      q.kb += n;
+      while (q.kb >= num_k && q.tile < total) {
+        q.kb -= num_k;
+        q.tile += nclusters;
+        if (q.tile < total) tile_coords(q.tile, p.tiles_m, p.tiles_n, q.tm, q.tn);
+      }
+    };
+    Pos cur{cluster, 0, 0, 0};
+    if (cur.tile < total) tile_coords(cur.tile, p.tiles_m, p.tiles_n, cur.tm, cur.tn);
+    step_by(cur, group);
+    Pos ahead = cur;
+    auto scale_at = [&](const Pos &q) -> uint32_t {
+      if (q.tile >= total) return 0u;
+      int64_t n, k;
+      pair_unit_coords<MODE>(u, static_cast<int64_t>(q.tn) * C::kTile + 128 * rank, q.kb, n, k);
+      return load_unit_scale<FMT>(p, n, k);
+    };
+    uint32_t sc[kD];
+#pragma unroll
+    for (int d = 0; d < kD; ++d) {
+      sc[d] = scale_at(ahead);
+      step_by(ahead, kG);
+    }
+    // unit geometry inside the stage (fixed for the thread)
+    uint32_t c_off, b_off[4];
+    if (MODE == MODE_FWD) {
+      const int r = u >> 1, h = u & 1;
+      c_off = r * 32 + h * 16;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) b_off[c] = (r >> 3) * 1024 + (r & 7) * 128 + (((4 * h + c) ^ (r & 7)) << 4);
+    } else {
+      const int j = (u & 7) + 8 * (u >> 5), part = (u >> 3) & 3;
+      c_off = j * 64 + ((part ^ ((j >> 1) & 3)) << 4);
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        b_off[c] = (part >> 1) * (kBK * 128) + j * 128 + (((4 * (part & 1) + c) ^ (j & 7)) << 4);
+    }
+    int it = group;
+    bool ok = true;
+    while (cur.tile < total && ok) {
+#pragma unroll
+      for (int d = 0; d < kD; ++d) {
+        if (cur.tile >= total || !ok) break;
+        const int s = it % S;
+        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+        if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
+        ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+        __syncwarp();
+        if (!ok) break;
+        uint32_t sc_lo, sc_hi;
+        if (FMT == 0) {
+          sc_lo = scale_bf16x2<0>(sc[d] & 0xFFu);
+          sc_hi = scale_bf16x2<0>(sc[d] >> 8);
+        } else {
+          sc_lo = sc_hi = scale_bf16x2<1>(sc[d]);
+        }
+        const uint4 cw = lds128(smem_u32(stage_c(s)) + c_off);
+        const uint32_t b_base = smem_u32(stage_b(s));
+        const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[4];
+          e2m1x8_to_bf16(words[c], o);
+          const uint32_t scv = c < 2 ? sc_lo : sc_hi;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
+          st_shared_v4(b_base + b_off[c], o[0], o[1], o[2], o[3]);
+        }
+        fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bready[s]);
+        sc[d] = scale_at(ahead);
+        step_by(ahead, kG);
+        step_by(cur, kG);
+        it += kG;
+      }
+    }
+  } else {
+    // ------------------------------------------------------ epilogue (warps 0-3, both CTAs)
+    const int r = warp * 32 + lane;
+    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
+    const float scale = FMT == 0 ? p.ws2 : 1.0f;
+    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
+    int tc = 0;
+    for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
+      int tm, tn;
+      tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+      const int64_t grow = static_cast<int64_t>(tm) * C::kTile + 128 * rank + r;
+      const int64_t col0 = static_cast<int64_t>(tn) * C::kTile;
+      const int ab = tc & 1;
+      const uint32_t au = static_cast<uint32_t>(tc >> 1);
+      if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
+      tc_fence_after();
+      const uint32_t t_buf = t_row + ab * kTmemCols;
+      for (int c0 = 0; c0 < C::kTile; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(t_buf + c0, v);
+        tmem_ld_wait();
+        if (grow >= p.M) continue;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int64_t gc = col0 + c0 + 8 * q;
+          if (gc >= Ng) continue;
+          uint32_t packed[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v[8 * q + 2 * e]) * scale,
+                                                            __uint_as_float(v[8 * q + 2 * e + 1]) * scale);
+            packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
+          }
+          *reinterpret_cast<uint4 *>(out + grow * Ng + gc) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[ab]), 0));
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync_all();
+  if (warp == C::kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, 2 * kTmemCols);
+  }
+}
+
+template <int MODE, int FMT>
+cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmC, int sm_count,
+                        cudaStream_t stream) {
+  using C = PairCfg;
+  static int attr_done_mask = 0;
+  static int max_clusters[32] = {0};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  auto kernel = sq_gemm_pair_kernel<MODE, FMT>;
+  if (!(attr_done_mask & (1 << (dev & 31)))) {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (sm_count / 2), 1, 1);
+    cfg.blockDim = dim3(C::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = sm_count / 2;
+    }
+    max_clusters[dev & 31] = n;
+    attr_done_mask |= 1 << (dev & 31);
+  }
+  const int64_t Ng = MODE == MODE_FWD ? a.N : a.K;
+  KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err,
+            static_cast<int>((a.M + C::kTile - 1) / C::kTile), static_cast<int>((Ng + C::kTile - 1) / C::kTile)};
+  const int64_t total = static_cast<int64_t>(p.tiles_m) * p.tiles_n;
+  const int64_t nc = total < max_clusters[dev & 31] ? total : max_clusters[dev & 31];
+  kernel<<<static_cast<unsigned>(2 * nc), C::kThreads, C::kSmemBytes, stream>>>(tmA, tmC, p);
+  return cudaGetLastError();
+}
+
 template <int MODE, int FMT>
 cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
                        cudaStream_t stream) {
@@ -685,12 +1136,12 @@ cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensor
 cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
                         cudaStream_t stream) {
   if (a.fmt == 0) {
-    if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 0>(a, tmA, tmB, sm_count, stream);
-    if (a.mode == MODE_DX) return launch_one<MODE_DX, 0>(a, tmA, tmB, sm_count, stream);
+    if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 0>(a, tmA, tmB, sm_count, stream);
+    if (a.mode == MODE_DX) return launch_pair<MODE_DX, 0>(a, tmA, tmB, sm_count, stream);
     return launch_one<MODE_SGRAD, 0>(a, tmA, tmB, sm_count, stream);
   }
-  if (a.mode == MODE_FWD) return launch_one<MODE_FWD, 1>(a, tmA, tmB, sm_count, stream);
-  if (a.mode == MODE_DX) return launch_one<MODE_DX, 1>(a, tmA, tmB, sm_count, stream);
+  if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 1>(a, tmA, tmB, sm_count, stream);
+  if (a.mode == MODE_DX) return launch_pair<MODE_DX, 1>(a, tmA, tmB, sm_count, stream);
   return launch_one<MODE_SGRAD, 1>(a, tmA, tmB, sm_count, stream);
 }
 
