@@ -4,21 +4,19 @@
 //   MODE_DX    dX[m,k] = sum_n dY[m,n] W[n,k]       its input gradient
 //   MODE_SGRAD g[n,b]  = sum_{k in b} code[n,k] sum_m dY[m,n] X[m,k]   its scale gradient
 //
-// with W[n,k] = code[n,k] * s[n, k/B] (Sec. 2). Persistent CTAs (one per SM)
-// walk 128 x 256 output tiles in an L2-friendly grouped order. Each tile
-// accumulates in one of two 256-column fp32 buffers in tensor memory (TMEM),
-// so the epilogue of one tile overlaps the mainloop of the next. Roles:
-//   warps 0-3   epilogue: tcgen05.ld (one TMEM lane = one output row per thread),
-//               ws2 scaling and bf16 stores (FWD/DX); code x dW products summed
-//               per block, mask, fp32 stores (SGRAD) -- dW never reaches HBM.
-//   warps 4-11  (FWD/DX) decode: the TMA-staged packed-code tile plus the scale
-//               bytes -> bf16 operand tile written straight into the 128B-swizzled
-//               smem layout the tensor core reads (K-major for FWD, MN-major for DX).
-//   next warp   TMA producer: activation tiles (and code tiles) into a 4-stage ring.
-//   last warp   TMEM allocator and the single MMA-issuing thread (tcgen05.mma,
-//               kind::f16, bf16 operands, fp32 accumulation).
-// For MODE_SGRAD both operands are MN-major TMA tiles (dY^T and X, contraction
-// over tokens) and there are no decode warps.
+// with W[n,k] = code[n,k] * s[n, k/B] (Sec. 2). All kernels are persistent
+// (one CTA per SM, tiles walked in an L2-friendly grouped order) and keep two
+// 256-column fp32 accumulators in tensor memory (TMEM), so the epilogue of one
+// tile overlaps the mainloop of the next.
+//
+// FWD / DX (sq_gemm_pair_kernel): a cluster of two CTAs computes a 256 x 256
+// tile with tcgen05.mma.cta_group::2. Each CTA streams its 128 activation rows
+// and its half of the packed-code tile by TMA, and 16 decode warps turn nibbles
+// and scale bytes into the bf16 weight operand directly in the 128B-swizzled
+// shared-memory layout the tensor core reads (K-major for FWD, MN-major for DX).
+//
+// SGRAD (sq_sgrad_kernel): one CTA per 128 x 256 tile of dW = dY^T X with both
+// operands as MN-major TMA tiles; the epilogue reduces code x dW per block.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA records
 // kErrWaitTimeout in the device error word, stops issuing, drains what it has
@@ -291,7 +289,7 @@ __device__ __forceinline__ uint32_t scale_bf16x2(uint32_t byte) {
   return u | (u << 16);
 }
 
-// ------------------------------------------------------------- the kernel
+// ------------------------------------------------------------- shared pieces
 
 struct KParams {
   const uint8_t *codes;
@@ -304,38 +302,18 @@ struct KParams {
   int tiles_m, tiles_n;
 };
 
-#ifndef SQ_DECODE_WARPS
-#define SQ_DECODE_WARPS 16
-#endif
-static_assert(512 % (32 * SQ_DECODE_WARPS) == 0, "decode warps must divide the 512 units of a k-step");
+// Tuning constants of the decode warps (compile-time; the defaults are the measured best).
 #ifndef SQ_PAIR_DEC_GROUPS
-#define SQ_PAIR_DEC_GROUPS 2
+#define SQ_PAIR_DEC_GROUPS 2  // groups of 8 decode warps per CTA, taking k-steps in turn
 #endif
 #ifndef SQ_SCALE_DEPTH
-#define SQ_SCALE_DEPTH 4
+#define SQ_SCALE_DEPTH 4      // scale bytes are loaded this many of a group's k-steps ahead
 #endif
-
-template <int MODE>
-struct Cfg {
-  static constexpr bool kDecode = MODE != MODE_SGRAD;
-  static constexpr int kEpiWarps = 4;                      // warps 0-3: TMEM lanes 0-127
-  static constexpr int kDecWarps = kDecode ? SQ_DECODE_WARPS : 0;  // warps 4 .. 3 + kDecWarps
-  static constexpr int kUnits = kDecode ? 512 / (32 * (kDecode ? kDecWarps : 1)) : 1;  // 32-weight units per thread per k-step
-  static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
-  static constexpr int kMmaWarp = kTmaWarp + 1;
-  static constexpr int kThreads = 32 * (kMmaWarp + 1);
-  static constexpr int kCStageBytes = kDecode ? 8192 : 0;  // packed-code tile (256 x 64 or 64 x 256 nibbles)
-  static constexpr int kStageBytes = kAStageBytes + kBStageBytes + kCStageBytes;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
-  static constexpr uint32_t kTxBytes =
-      MODE == MODE_SGRAD ? kAStageBytes + kBStageBytes : kAStageBytes + kCStageBytes;
-};
 
 // Persistent tile order: tiles are walked in groups of kGroup row-tiles, the
 // column index varying slowest inside a group, so the CTAs resident at any
 // moment share a few row panels and column panels in L2.
 constexpr int kGroup = 8;
-
 
 __device__ __forceinline__ void tile_coords(int id, int tiles_m, int tiles_n, int &tm, int &tn) {
   const int per_group = kGroup * tiles_n;
@@ -364,30 +342,35 @@ __device__ __forceinline__ uint32_t load_unit_scale(const KParams &p, int64_t n,
   return __ldg(p.scales + n * G + k / 32);
 }
 
-// Weight coordinates (n, k) of decode unit u (0..511) of a k-step.
-template <int MODE>
-__device__ __forceinline__ void unit_coords(int u, int64_t col0, int kb, int64_t &n, int64_t &k) {
-  if (MODE == MODE_FWD) {  // 256 rows (out features) x 64 k: unit = half a row
-    n = col0 + (u >> 1);
-    k = static_cast<int64_t>(kb) * kBK + 32 * (u & 1);
-  } else {  // 64 contraction rows (out features) x 256 k: unit = an eighth of a row
-    n = static_cast<int64_t>(kb) * kBK + (u & 7) + 8 * (u >> 6);
-    k = col0 + 32 * ((u >> 3) & 7);
-  }
-}
+// ------------------------------------------------------------- scale-gradient kernel
+//
+// D[n, k] = sum_m dY[m, n] X[m, k] on one CTA per SM: both operands are MN-major
+// TMA tiles (dY^T as two 64(n) x 64(m) boxes, X as four 64(k) x 64(m) boxes),
+// contraction over the tokens. The epilogue multiplies each dW element by its
+// E2M1 code and sums every block of B columns, applies the STE mask and writes
+// g[n, b]; the dW tile never leaves the SM.
 
-template <int MODE, int FMT>
-__global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
-    sq_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const KParams p) {
-  using C = Cfg<MODE>;
+struct SgradCfg {
+  static constexpr int kEpiWarps = 4;  // warps 0-3: TMEM lanes 0-127
+  static constexpr int kTmaWarp = 4;
+  static constexpr int kMmaWarp = 5;
+  static constexpr int kThreads = 192;
+  static constexpr int kStageBytes = kAStageBytes + kBStageBytes;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+};
+
+template <int FMT>
+__global__ void __launch_bounds__(SgradCfg::kThreads, 1)
+    sq_sgrad_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const KParams p) {
+  using C = SgradCfg;
+  constexpr int B = FMT == 0 ? 16 : 32;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * C::kStageBytes);
   uint64_t *afull = bars;                 // TMA tiles of the stage landed      (1 arrival + tx)
-  uint64_t *bfull = bars + kStages;       // decoded B tile written             (kDecWarps arrivals)
-  uint64_t *empty = bars + 2 * kStages;   // MMAs reading the stage completed   (tcgen05.commit)
-  uint64_t *tfull = bars + 3 * kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
+  uint64_t *empty = bars + kStages;       // MMAs reading the stage completed   (tcgen05.commit)
+  uint64_t *tfull = bars + 2 * kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
   uint64_t *tempty = tfull + 2;           // [2] accumulator buffer drained     (kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
@@ -396,17 +379,14 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int total = p.tiles_m * p.tiles_n;
-  const int64_t Kg = MODE == MODE_FWD ? p.K : (MODE == MODE_DX ? p.N : p.M);
-  const int num_k = static_cast<int>((Kg + kBK - 1) / kBK);
+  const int num_k = static_cast<int>((p.M + kBK - 1) / kBK);
 
   auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
   auto stage_b = [&](int s) { return smem + s * C::kStageBytes + kAStageBytes; };
-  auto stage_c = [&](int s) { return smem + s * C::kStageBytes + kAStageBytes + kBStageBytes; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&afull[s], 1);
-      mbar_init(&bfull[s], C::kDecWarps > 0 ? C::kDecWarps : 1);
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -440,22 +420,12 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           const int s = it % kStages;
           const uint32_t use = static_cast<uint32_t>(it / kStages);
           if (it >= kStages && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
-          mbar_arrive_expect_tx(&afull[s], C::kTxBytes);
+          mbar_arrive_expect_tx(&afull[s], C::kStageBytes);
           const uint32_t a_dst = smem_u32(stage_a(s));
+          const uint32_t b_dst = smem_u32(stage_b(s));
           const int32_t kc = kb * kBK;
-          if (MODE == MODE_SGRAD) {
-            const uint32_t b_dst = smem_u32(stage_b(s));
-            // dY^T tile: two 64(n) x 64(m) boxes; X tile: four 64(k) x 64(m) boxes (MN-major).
-            for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * (kBK * 128), &tmA, &afull[s], row0 + 64 * j, kc);
-            for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * (kBK * 128), &tmB, &afull[s], col0 + 64 * j, kc);
-          } else {
-            const uint32_t c_dst = smem_u32(stage_c(s));
-            tma_load_2d(a_dst, &tmA, &afull[s], kc, row0);
-            if (MODE == MODE_FWD)  // codes [N, K/2]: 256 rows x 32 bytes at (byte k/2, row n)
-              tma_load_2d(c_dst, &tmB, &afull[s], kc / 2, col0);
-            else                   // 64 rows x 128 bytes, 128-byte swizzle
-              tma_load_2d(c_dst, &tmB, &afull[s], col0 / 2, kc);
-          }
+          for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * (kBK * 128), &tmA, &afull[s], row0 + 64 * j, kc);
+          for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * (kBK * 128), &tmB, &afull[s], col0 + 64 * j, kc);
         }
       }
       if (*abort_flag) {
@@ -467,7 +437,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(kBM, kBN, MODE == MODE_SGRAD ? 1 : 0, MODE == MODE_FWD ? 0 : 1);
+      constexpr uint32_t idesc = idesc_bf16(kBM, kBN, 1, 1);
       int it = 0, tc = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tc) {
@@ -479,18 +449,13 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         for (int kb = 0; kb < num_k; ++kb, ++it) {
           const int s = it % kStages;
           const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-          ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
-          if (ok && C::kDecode) ok = mbar_wait(&bfull[s], ph, abort_flag, p.err);
-          if (!ok) break;
-          tc_fence_after();
+          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
           const uint32_t a_base = smem_u32(stage_a(s));
           const uint32_t b_base = smem_u32(stage_b(s));
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = MODE == MODE_SGRAD ? smem_desc_sw128(a_base + kk * 2048, kBK * 128, 1024)
-                                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
-            const uint64_t bd = MODE == MODE_FWD ? smem_desc_sw128(b_base + kk * 32, 16, 1024)
-                                                 : smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
+            const uint64_t ad = smem_desc_sw128(a_base + kk * 2048, kBK * 128, 1024);
+            const uint64_t bd = smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
             umma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit(&empty[s]);
@@ -500,187 +465,58 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       umma_commit(drain);  // completes once every MMA issued above has finished
       mbar_drain(drain, 0);
     }
-  } else if (warp >= C::kEpiWarps) {
-    // ------------------------------------------------------ decode (FWD / DX)
-    if (C::kDecode) {
-      constexpr int kDecThreads = 32 * C::kDecWarps;
-      constexpr int kU = C::kUnits;
-      constexpr int kD = SQ_SCALE_DEPTH;  // scale bytes are loaded kD k-steps ahead (codes arrive by TMA)
-      const int dt = threadIdx.x - 32 * C::kEpiWarps;  // this thread owns units dt + kDecThreads * i
-      // position in the flattened (tile, k-step) walk: current and kD steps ahead
-      int c_tile = blockIdx.x, c_kb = 0, c_tn = 0, c_tm = 0;
-      if (c_tile < total) tile_coords(c_tile, p.tiles_m, p.tiles_n, c_tm, c_tn);
-      int a_tile = c_tile, a_kb = 0, a_tn = c_tn, a_tm = c_tm;
-      auto advance = [&](int &tile, int &kb, int &tm, int &tn) {
-        if (++kb == num_k) {
-          kb = 0;
-          tile += gridDim.x;
-          if (tile < total) tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-        }
-      };
-      uint32_t sc[kD][kU];
-#pragma unroll
-      for (int d = 0; d < kD; ++d) {
-#pragma unroll
-        for (int i = 0; i < kU; ++i) {
-          int64_t n, k;
-          unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(a_tn) * kBN, a_kb, n, k);
-          sc[d][i] = a_tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
-        }
-        advance(a_tile, a_kb, a_tm, a_tn);
-      }
-      int it = 0;
-      bool ok = true;
-      while (c_tile < total && ok) {
-#pragma unroll
-        for (int d = 0; d < kD; ++d) {
-          if (c_tile >= total || !ok) break;
-          const int s = it % kStages;
-          const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-          // one lane polls the barrier (32 polling lanes serialise), the warp follows
-          if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
-          ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
-          __syncwarp();
-          if (!ok) break;
-          const uint32_t b_base = smem_u32(stage_b(s));
-          const uint32_t c_base = smem_u32(stage_c(s));
-#pragma unroll
-          for (int i = 0; i < kU; ++i) {
-            const int u = dt + kDecThreads * i;
-            uint32_t sc_lo, sc_hi;
-            if (FMT == 0) {
-              sc_lo = scale_bf16x2<0>(sc[d][i] & 0xFFu);
-              sc_hi = scale_bf16x2<0>(sc[d][i] >> 8);
-            } else {
-              sc_lo = sc_hi = scale_bf16x2<1>(sc[d][i]);
-            }
-            uint4 cw;
-            if (MODE == MODE_FWD) {
-              cw = lds128(c_base + (u >> 1) * 32 + (u & 1) * 16);
-            } else {
-              const int j = (u & 7) + 8 * (u >> 6);
-              const int part = (u >> 3) & 7;
-              cw = lds128(c_base + j * 128 + ((part ^ (j & 7)) << 4));
-            }
-            const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-              uint32_t o[4];
-              e2m1x8_to_bf16(words[c], o);
-              const uint32_t scv = c < 2 ? sc_lo : sc_hi;
-#pragma unroll
-              for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
-              uint32_t addr;
-              if (MODE == MODE_FWD) {
-                const int r = u >> 1;
-                const int chunk = 4 * (u & 1) + c;
-                addr = b_base + (r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4);
-              } else {
-                const int j = (u & 7) + 8 * (u >> 6);
-                const int part = (u >> 3) & 7;
-                const int chunk = 4 * (part & 1) + c;
-                addr = b_base + (part >> 1) * (kBK * 128) + j * 128 + ((chunk ^ (j & 7)) << 4);
-              }
-              st_shared_v4(addr, o[0], o[1], o[2], o[3]);
-            }
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bfull[s]);
-          // refill this ring slot with the scales of the position kD steps ahead
-#pragma unroll
-          for (int i = 0; i < kU; ++i) {
-            int64_t n, k;
-            unit_coords<MODE>(dt + kDecThreads * i, static_cast<int64_t>(a_tn) * kBN, a_kb, n, k);
-            sc[d][i] = a_tile < total ? load_unit_scale<FMT>(p, n, k) : 0u;
-          }
-          advance(a_tile, a_kb, a_tm, a_tn);
-          advance(c_tile, c_kb, c_tm, c_tn);
-          ++it;
-        }
-      }
-    }
   } else {
     // ------------------------------------------------------ epilogue (warps 0-3)
     const int r = warp * 32 + lane;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const int64_t G = p.K / B;
+    float *g = static_cast<float *>(p.out);
     int tc = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++tc) {
       int tm, tn;
       tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-      const int64_t row0 = static_cast<int64_t>(tm) * kBM, col0 = static_cast<int64_t>(tn) * kBN;
+      const int64_t n = static_cast<int64_t>(tm) * kBM + r;
+      const int64_t col0 = static_cast<int64_t>(tn) * kBN;
       const int ab = tc & 1;
       const uint32_t au = static_cast<uint32_t>(tc >> 1);
       if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
       tc_fence_after();
       const uint32_t t_buf = t_row + ab * kTmemCols;
-      if (MODE != MODE_SGRAD) {
-        const int64_t Mg = p.M;
-        const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
-        const int64_t grow = row0 + r;
-        const float scale = FMT == 0 ? p.ws2 : 1.0f;
-        __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
-        for (int c0 = 0; c0 < kBN; c0 += 32) {
-          uint32_t v[32];
-          tmem_ld32(t_buf + c0, v);
-          tmem_ld_wait();
-          if (grow >= Mg) continue;
+      for (int c0 = 0; c0 < kBN; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(t_buf + c0, v);
+        tmem_ld_wait();
+        const int64_t k = col0 + c0;
+        if (n >= p.N || k >= p.K) continue;
+        const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
+        const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+        float part[4];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int64_t gc = col0 + c0 + 8 * q;
-            if (gc >= Ng) continue;
-            uint32_t packed[4];
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[4];
+          e2m1x8_to_bf16(words[c], o);
+          float acc = 0.f;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float a = __uint_as_float(v[8 * q + 2 * e]) * scale;
-              const float b = __uint_as_float(v[8 * q + 2 * e + 1]) * scale;
-              const __nv_bfloat162 h2 = __floats2bfloat162_rn(a, b);
-              packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
-            }
-            *reinterpret_cast<uint4 *>(out + grow * Ng + gc) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+          for (int e = 0; e < 4; ++e) {
+            acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
+            acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
           }
+          part[c] = acc;
         }
-      } else {
-        constexpr int B = FMT == 0 ? 16 : 32;
-        const int64_t n = row0 + r;
-        const int64_t G = p.K / B;
-        float *g = static_cast<float *>(p.out);
-        for (int c0 = 0; c0 < kBN; c0 += 32) {
-          uint32_t v[32];
-          tmem_ld32(t_buf + c0, v);
-          tmem_ld_wait();
-          const int64_t k = col0 + c0;
-          if (n >= p.N || k >= p.K) continue;
-          const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
-          const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
-          float part[4];
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            uint32_t o[4];
-            e2m1x8_to_bf16(words[c], o);
-            float acc = 0.f;
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
-              acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
-            }
-            part[c] = acc;
+        if (FMT == 0) {
+          const int64_t b = k / 16;
+          float g0 = part[0] + part[1];
+          float g1 = part[2] + part[3];
+          if (p.mask) {
+            g0 *= static_cast<float>(p.mask[n * G + b]);
+            g1 *= static_cast<float>(p.mask[n * G + b + 1]);
           }
-          if (FMT == 0) {
-            const int64_t b = k / 16;
-            float g0 = part[0] + part[1];
-            float g1 = part[2] + part[3];
-            if (p.mask) {
-              g0 *= static_cast<float>(p.mask[n * G + b]);
-              g1 *= static_cast<float>(p.mask[n * G + b + 1]);
-            }
-            *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
-          } else {
-            const int64_t b = k / 32;
-            float g0 = (part[0] + part[1]) + (part[2] + part[3]);
-            if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
-            g[n * G + b] = g0;
-          }
+          *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
+        } else {
+          const int64_t b = k / 32;
+          float g0 = (part[0] + part[1]) + (part[2] + part[3]);
+          if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
+          g[n * G + b] = g0;
         }
       }
       tc_fence_before();
@@ -899,7 +735,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           ok = mbar_wait(&bready[s], ph, abort_flag, p.err);                // own half
           if (ok) ok = mbar_wait_cluster(&pready[s], ph, abort_flag, p.err);  // the peer's half
           if (!ok) break;
-          tc_fence_after();
           const uint32_t a_base = smem_u32(stage_a(s));
           const uint32_t b_base = smem_u32(stage_b(s));
 #pragma unroll
@@ -1108,26 +943,24 @@ cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
   return cudaGetLastError();
 }
 
-template <int MODE, int FMT>
-cudaError_t launch_one(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
-                       cudaStream_t stream) {
-  using C = Cfg<MODE>;
+template <int FMT>
+cudaError_t launch_sgrad(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
+                         cudaStream_t stream) {
+  using C = SgradCfg;
   static int attr_done_mask = 0;  // per device ordinal (first 31)
   int dev = 0;
   cudaGetDevice(&dev);
   if (!(attr_done_mask & (1 << (dev & 31)))) {
-    cudaError_t e = cudaFuncSetAttribute(sq_gemm_kernel<MODE, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(sq_sgrad_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          C::kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_done_mask |= 1 << (dev & 31);
   }
-  const int64_t Mg = MODE == MODE_SGRAD ? a.N : a.M;
-  const int64_t Ng = MODE == MODE_FWD ? a.N : a.K;
   KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err,
-            static_cast<int>((Mg + kBM - 1) / kBM), static_cast<int>((Ng + kBN - 1) / kBN)};
+            static_cast<int>((a.N + kBM - 1) / kBM), static_cast<int>((a.K + kBN - 1) / kBN)};
   const int64_t total = static_cast<int64_t>(p.tiles_m) * p.tiles_n;
   const int grid = static_cast<int>(total < sm_count ? total : sm_count);
-  sq_gemm_kernel<MODE, FMT><<<grid, C::kThreads, C::kSmemBytes, stream>>>(tmA, tmB, p);
+  sq_sgrad_kernel<FMT><<<grid, C::kThreads, C::kSmemBytes, stream>>>(tmA, tmB, p);
   return cudaGetLastError();
 }
 
@@ -1138,11 +971,11 @@ cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
   if (a.fmt == 0) {
     if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 0>(a, tmA, tmB, sm_count, stream);
     if (a.mode == MODE_DX) return launch_pair<MODE_DX, 0>(a, tmA, tmB, sm_count, stream);
-    return launch_one<MODE_SGRAD, 0>(a, tmA, tmB, sm_count, stream);
+    return launch_sgrad<0>(a, tmA, tmB, sm_count, stream);
   }
   if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 1>(a, tmA, tmB, sm_count, stream);
   if (a.mode == MODE_DX) return launch_pair<MODE_DX, 1>(a, tmA, tmB, sm_count, stream);
-  return launch_one<MODE_SGRAD, 1>(a, tmA, tmB, sm_count, stream);
+  return launch_sgrad<1>(a, tmA, tmB, sm_count, stream);
 }
 
 }  // namespace sqi
