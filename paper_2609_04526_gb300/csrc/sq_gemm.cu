@@ -561,6 +561,15 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   return r;
 }
 
+// Asynchronous 4-byte store into another CTA's shared memory that completes 4
+// bytes of transaction on that CTA's mbarrier; the complete-tx has release
+// semantics at cluster scope and the issuing thread does not wait for it.
+__device__ __forceinline__ void st_async_signal(uint32_t cluster_dst, uint32_t cluster_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.u32 [%0], %1, [%2];" ::"r"(cluster_dst), "r"(1u),
+               "r"(cluster_bar)
+               : "memory");
+}
+
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
@@ -608,15 +617,14 @@ struct PairCfg {
   static constexpr int kDecWarps = 8 * kDecGroups;       // 8 warps per group: one 32-weight unit per thread
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
   static constexpr int kMmaWarp = kTmaWarp + 1;
-  static constexpr int kSigWarp0 = kMmaWarp + 1;
-  static constexpr int kSigWarps = 4;    // peer CTA: forward "half decoded" to the leader, k-steps in turn
-  static constexpr int kThreads = 32 * (kSigWarp0 + kSigWarps);
+  static constexpr int kThreads = 32 * (kMmaWarp + 1);
+  static constexpr uint32_t kSignalBytes = 4 * 16;  // st.async bytes per stage: 8 decode warps x 2 CTAs
   static constexpr int kStages = 6;
   static constexpr int kA = 128 * kBK * 2;  // 16 KiB: this CTA's 128 activation rows
   static constexpr int kB = 128 * kBK * 2;  // 16 KiB: this CTA's half of the decoded weight tile
   static constexpr int kC = 4096;           // packed codes of that half
   static constexpr int kStageBytes = kA + kB + kC;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 512;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 1024;
   static constexpr uint32_t kTx = kA + kC;
   static constexpr int kTile = 256;         // output tile is kTile x kTile per pair
 };
@@ -643,14 +651,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + S * C::kStageBytes);
   uint64_t *afull = bars;             // this CTA's TMA tiles landed            (1 arrival + tx)
-  uint64_t *bready = bars + S;        // this CTA's weight half decoded          (8 decode-warp arrivals)
-  uint64_t *empty = bars + 2 * S;     // pair MMAs reading the stage completed   (multicast commit)
-  uint64_t *pready = bars + 3 * S;    // leader: the peer's half decoded         (1 cluster arrival)
-  uint64_t *tfull = bars + 4 * S;     // [2] accumulator buffer complete         (multicast commit)
+  uint64_t *empty = bars + S;         // pair MMAs reading the stage completed   (multicast commit)
+  uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded      (1 arrival + st.async tx)
+  uint64_t *tfull = bars + 3 * S;     // [2] accumulator buffer complete         (multicast commit)
   uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained      (2 x kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // [S][2][8] leader: st.async targets
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -668,7 +676,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&afull[s], 1);
-      mbar_init(&bready[s], 8);  // one arrival per decode warp of the group that owns the k-step
       mbar_init(&empty[s], 1);
       mbar_init(&pready[s], 1);
     }
@@ -705,6 +712,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           const uint32_t use = static_cast<uint32_t>(it / S);
           if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
           mbar_arrive_expect_tx(&afull[s], C::kTx);
+          if (rank == 0) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
           tma_load_2d(smem_u32(stage_a(s)), &tmA, &afull[s], kb * kBK, row0);
           if (MODE == MODE_FWD)  // codes: 128 rows x 32 bytes
             tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], kb * (kBK / 2), half0);
@@ -732,9 +740,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         for (int kb = 0; kb < num_k; ++kb, ++it) {
           const int s = it % S;
           const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
-          ok = mbar_wait(&bready[s], ph, abort_flag, p.err);                // own half
-          if (ok) ok = mbar_wait_cluster(&pready[s], ph, abort_flag, p.err);  // the peer's half
-          if (!ok) break;
+          if (!(ok = mbar_wait_cluster(&pready[s], ph, abort_flag, p.err))) break;  // both halves decoded
           const uint32_t a_base = smem_u32(stage_a(s));
           const uint32_t b_base = smem_u32(stage_b(s));
 #pragma unroll
@@ -750,22 +756,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       }
       umma_commit_pair(drain);
       mbar_drain(drain, 0);
-    }
-  } else if (warp >= C::kSigWarp0) {
-    // ------------------------------------------------------ signal warps (peer CTA)
-    // Forward "this CTA's weight half of stage s is decoded" to the leader with
-    // one cluster-scope release per k-step. A cluster-scope release holds the
-    // issuing warp for a long time, so it is kept off the decode warps and the
-    // k-steps are spread over kSigWarps warps.
-    if (rank == 1 && lane == 0) {
-      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
-      const int iters = my_tiles * num_k;
-      const uint32_t leader_pready = mapa_shared(smem_u32(&pready[0]), 0);
-      for (int it = warp - C::kSigWarp0; it < iters; it += C::kSigWarps) {
-        const int s = it % S;
-        if (!mbar_wait(&bready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
-        mbar_arrive_cluster(leader_pready + 8u * s);
-      }
     }
   } else if (warp >= C::kEpiWarps) {
     // ------------------------------------------------------ decode (both CTAs)
@@ -851,7 +841,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         }
         fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bready[s]);
+        // tell the leader without waiting: an async store whose complete-tx on the
+        // leader's stage barrier is a cluster-scope release (both CTAs, 16 warps per stage)
+        if (lane == 0)
+          st_async_signal(mapa_shared(smem_u32(&sink[(s * 2 + rank) * 8 + dw % 8]), 0),
+                          mapa_shared(smem_u32(&pready[s]), 0));
         sc[d] = scale_at(ahead);
         step_by(ahead, kG);
         step_by(cur, kG);
