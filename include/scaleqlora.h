@@ -132,6 +132,29 @@ sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, floa
 sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
                    uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream);
 
+/* Allocation-free variant of sq_scale_grad. The paper has no counterpart: this
+ * entry point exists for callers of this library that cannot call cudaMalloc --
+ * code whose device memory is owned by an outside pool or allocator that must
+ * account for every byte, and hot loops that cannot accept the device-wide
+ * synchronisation cudaMalloc / cudaFree may cause. It takes no handle and
+ * allocates nothing: the kernel's scratch (the device error word its bounded
+ * waits set) lives in a file-scope static __device__ array of 256 bytes that
+ * every GPU loading the library holds until the process exits.
+ *  - Arguments, layouts and results are those of sq_scale_grad.
+ *  - Scratch limit: 256 bytes; this kernel needs one 4-byte word for any M, N, K,
+ *    and a call whose need exceeded the array would return SQ_ERR_INVALID_ARG.
+ *  - The first call on each device sets up (checks the device, looks up the
+ *    array's device address with cudaGetSymbolAddress); make that first call
+ *    before any stream capture.
+ *  - Every call on a device shares the array: the error word is cleared at the
+ *    start of each call, and calls that overlap on the GPU race on it.
+ *  - device_status: device int32 or NULL; if given, it receives the error word
+ *    after the kernel (0, or nonzero when a bounded device wait ran out).
+ * Returns SQ_OK, SQ_ERR_INVALID_ARG, SQ_ERR_UNSUPPORTED, SQ_ERR_DEVICE or
+ * SQ_ERR_CUDA; there is no handle, so no error text. */
+sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
+                                const uint8_t *mask, float *g, int32_t *device_status, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -26,7 +26,7 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 
 # Every entry point the header declares (checked against include/scaleqlora.h by the tests).
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
-           "sq_scale_grad", "sq_project_scales", "sq_merge")
+           "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_scale_grad_noalloc")
 
 
 class SQError(RuntimeError):
@@ -66,6 +66,7 @@ def load() -> ctypes.CDLL:
     L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
     L.sq_project_scales.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
     L.sq_merge.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
+    L.sq_scale_grad_noalloc.argtypes = [W, vp, vp, i64, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
