@@ -49,6 +49,22 @@ def parse_args():
     return ap.parse_args()
 
 
+def profiled_traffic(workload):
+    """DRAM bytes per launch measured by ncu for each kernel kind (profiles/), or
+    None for every kind when the kernel sources changed since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}_layer_step.json")
+    if not os.path.exists(path):
+        return {}
+    with open(path) as f:
+        prof = json.load(f)
+    for name, digest in prof.get("source_sha256", {}).items():
+        src = os.path.join(ROOT, "paper_2609_04526_gb300", "csrc", name)
+        if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != digest:
+            return {}
+    return prof.get("kernels", {})
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -145,14 +161,6 @@ class LayerState:
             st["qw"] = pkg.QuantWeight(wl.fmt, lin.N, lin.K, w.codes, st["qbytes"], w.ws2)
             self.lin.append(st)
 
-    def inputs(self):
-        """(name, tensor) of every per-step input: activations, output gradients, latent scales."""
-        out = [("X:" + k, v) for k, v in self.acts.items()]
-        for st in self.lin:
-            out.append(("dY:" + st["lin"].name, st["dY"]))
-            out.append(("L:" + st["lin"].name, st["latent"]))
-        return out
-
     def results(self):
         """(name, tensor) of the step's results read back by a user: scale gradients,
         merged scale planes and the NaN / changed-byte counters."""
@@ -163,27 +171,46 @@ class LayerState:
         return out
 
 
-def run_step(h, S, stream, events=None):
+def input_set(S):
+    """The step's inputs as a dict: activations by name, then dY and latent per linear."""
+    return {"acts": dict(S.acts), "dY": [st["dY"] for st in S.lin], "L": [st["latent"] for st in S.lin]}
+
+
+def clone_input_set(ins):
+    return {"acts": {k: torch.empty_like(v) for k, v in ins["acts"].items()},
+            "dY": [torch.empty_like(t) for t in ins["dY"]], "L": [torch.empty_like(t) for t in ins["L"]]}
+
+
+def flat_inputs(ins):
+    return list(ins["acts"].values()) + ins["dY"] + ins["L"]
+
+
+def run_step(h, S, stream, events=None, ins=None):
+    """One step over every linear: projection (+ STE mask), forward, input gradient,
+    masked scale gradient, merge into the artifact scale plane."""
     fmt = S.wl.fmt
+    ins = input_set(S) if ins is None else ins
     for i, st in enumerate(S.lin):
-        X = S.acts[st["lin"].x]
+        X = ins["acts"][st["lin"].x]
+        dY = ins["dY"][i]
+        L = ins["L"][i]
         ev = events[i] if events is not None else None
         if ev:
             ev[0].record(stream)
-        h.sq_project_scales(fmt, st["latent"], st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
+        h.sq_project_scales(fmt, L, st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
                             nonfinite=st["nonfinite"], stream=stream)
         if ev:
             ev[1].record(stream)
         h.sq_fwd(st["qw"], X, st["Y"], stream=stream)
         if ev:
             ev[2].record(stream)
-        h.sq_bwd_dx(st["qw"], st["dY"], st["dX"], stream=stream)
+        h.sq_bwd_dx(st["qw"], dY, st["dX"], stream=stream)
         if ev:
             ev[3].record(stream)
-        h.sq_scale_grad(st["qw"], X, st["dY"], mask=st["mask"], g=st["g"], stream=stream)
+        h.sq_scale_grad(st["qw"], X, dY, mask=st["mask"], g=st["g"], stream=stream)
         if ev:
             ev[4].record(stream)
-        h.sq_merge(fmt, st["latent"], st["ws2"], st["art"], changed=st["changed"], stream=stream)
+        h.sq_merge(fmt, L, st["ws2"], st["art"], changed=st["changed"], stream=stream)
         if ev:
             ev[5].record(stream)
 
@@ -337,33 +364,58 @@ def run_ours(args):
             ach = by[kind] / t / 1e9
             kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
     dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
+    traffic = profiled_traffic(wl.key)
+    for kind in KINDS:
+        if kind in traffic:
+            kernels[kind]["dram_bytes_per_launch"] = traffic[kind]["dram_bytes_per_launch"]
     value = flops_step * args.steps * world / (ms_total / 1e3) / 1e12
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API with host buffers: every step copies
+    # its inputs from pinned host memory and reads its results back; the copies of
+    # step k+1 run on a copy stream into a second input buffer set while step k
+    # computes.
     e2e = None
     if not args.no_e2e:
-        ins = [(n, t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for n, t in S.inputs()]
-        outs = [(n, t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for n, t in S.results()]
-        for _, dev, hst in ins:
+        sets = [input_set(S), clone_input_set(input_set(S))]
+        host_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in flat_inputs(sets[0])]
+        for hst, dev in zip(host_in, flat_inputs(sets[0])):
             hst.copy_(dev)
-        h2d = sum(t.numel() * t.element_size() for _, t, _ in ins)
-        d2h = sum(t.numel() * t.element_size() for _, t, _ in outs)
+        outs = [(t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for _, t in S.results()]
+        h2d = sum(t.numel() * t.element_size() for t in host_in)
+        d2h = sum(t.numel() * t.element_size() for t, _ in outs)
+        copy_stream = torch.cuda.Stream()
+        ready = [torch.cuda.Event(), torch.cuda.Event()]
+        free = [torch.cuda.Event(), torch.cuda.Event()]
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+        def issue_copy(k):
+            b = k % 2
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(free[b] if k >= 2 else e0)
+                for hst, dev in zip(host_in, flat_inputs(sets[b])):
+                    dev.copy_(hst, non_blocking=True)
+                ready[b].record(copy_stream)
+
         barrier(world)
         torch.cuda.synchronize()
         e0.record(stream)
-        for _ in range(args.steps):
-            for _, dev, hst in ins:
-                dev.copy_(hst, non_blocking=True)
-            run_step(h, S, stream)
-            for _, dev, hst in outs:
+        issue_copy(0)
+        for k in range(args.steps):
+            if k + 1 < args.steps:
+                issue_copy(k + 1)
+            stream.wait_event(ready[k % 2])
+            run_step(h, S, stream, ins=sets[k % 2])
+            free[k % 2].record(stream)
+            for dev, hst in outs:
                 hst.copy_(dev, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
         h.sq_sync(stream)
         e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
         e2e = {"value": flops_step * args.steps * world / (e2e_ms / 1e3) / 1e12, "unit": UNIT,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps,
+               "overlap": "inputs of step k+1 copied on a second stream while step k computes"}
+        del sets, host_in
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
@@ -388,7 +440,11 @@ def run_ours(args):
                        "parallelism": f"replicas x{world}", "flops_per_step": flops_step},
             "roofline": {"bound": "tensor", "kernel": dom, "achieved": k["achieved"],
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": k["achieved"] / pk["bf16_sustained"],
-                         "traffic": None, "peak_source": f"{pk['source']} bf16 sustained"},
+                         "traffic": traffic.get(dom, {}).get("dram_bytes_per_launch"),
+                         "algorithmic_bytes": traffic.get(dom, {}).get("algorithmic_bytes_per_launch"),
+                         "traffic_note": "ncu dram bytes per launch, mean over the layer's 7 launches of this kernel "
+                                         "(profiles/traffic_c5_layer_step.json); null if the kernels changed since",
+                         "peak_source": f"{pk['source']} bf16 sustained"},
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels,
             "e2e": e2e, "cpu_baseline": cpu,
