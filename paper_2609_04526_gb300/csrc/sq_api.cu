@@ -170,13 +170,13 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   const int64_t K2 = w->K / 2;  // code bytes per row
   if (mode == sqi::MODE_FWD) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));  // X, 128 x 64 K-major boxes
-    // codes: 128 rows x 32 bytes (64 weights) per k-step and CTA of the pair
-    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, sqi::kBK / 2, 128,
-                    CU_TENSOR_MAP_SWIZZLE_NONE));
+    // codes: 128 rows x 64 bytes (128 weights) per stage and CTA of the pair, 64-byte swizzle
+    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
+                    CU_TENSOR_MAP_SWIZZLE_64B));
   } else if (mode == sqi::MODE_DX) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));  // dY, 128 x 64 K-major boxes
-    // codes: 64 contraction rows x 64 bytes (128 weights) per k-step and CTA, 64-byte swizzle
-    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, sqi::kBK,
+    // codes: 128 contraction rows x 64 bytes (128 weights) per stage and CTA, 64-byte swizzle
+    SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
   } else {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBK));  // dY, MN-major boxes 64(n) x 64(m)

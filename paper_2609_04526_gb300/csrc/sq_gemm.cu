@@ -303,9 +303,6 @@ struct KParams {
 };
 
 // Tuning constants of the decode warps (compile-time; the defaults are the measured best).
-#ifndef SQ_PAIR_DEC_GROUPS
-#define SQ_PAIR_DEC_GROUPS 2  // groups of 8 decode warps per CTA, taking k-steps in turn
-#endif
 #ifndef SQ_SCALE_DEPTH
 #define SQ_SCALE_DEPTH 4      // scale bytes are loaded this many of a group's k-steps ahead
 #endif
@@ -436,29 +433,41 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer
+    // The next stage's barrier is polled between the MMAs of the current one
+    // (each tcgen05.mma blocks until the tensor core takes it).
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, kBN, 1, 1);
-      int it = 0, tc = 0;
-      bool ok = true;
+      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), kBK * 128, 1024);
+      const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), kBK * 128, 1024);
+      const int my_tiles = static_cast<int>(blockIdx.x) < total ? (total - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+      int left = my_tiles * num_k;
+      int s = 0;
+      uint32_t ph = 0;
+      int tc = 0;
+      bool ok = true, ready = false;
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tc) {
         const int ab = tc & 1;
         const uint32_t au = static_cast<uint32_t>(tc >> 1);
         if (tc >= 2 && !(ok = mbar_wait(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
-        for (int kb = 0; kb < num_k; ++kb, ++it) {
-          const int s = it % kStages;
-          const uint32_t ph = static_cast<uint32_t>(it / kStages) & 1u;
-          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
-          const uint32_t a_base = smem_u32(stage_a(s));
-          const uint32_t b_base = smem_u32(stage_b(s));
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!ready && !(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
+          const int ns = s + 1 == kStages ? 0 : s + 1;
+          const uint32_t nph = ns == 0 ? ph ^ 1u : ph;
+          --left;
+          ready = false;
+          const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
+          const uint64_t a0 = ad_base + so, b0 = bd_base + so;
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = smem_desc_sw128(a_base + kk * 2048, kBK * 128, 1024);
-            const uint64_t bd = smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
-            umma_bf16(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            umma_bf16(d_tmem, a0 + static_cast<uint64_t>(kk * 2048 >> 4), b0 + static_cast<uint64_t>(kk * 2048 >> 4),
+                      idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            if (left > 0 && !ready) ready = mbar_try_wait(&afull[ns], nph);
           }
           umma_commit(&empty[s]);
+          s = ns;
+          ph = nph;
         }
         if (ok) umma_commit(&tfull[ab]);
       }
@@ -613,31 +622,36 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t *bar) {
 
 struct PairCfg {
   static constexpr int kEpiWarps = 4;    // warps 0-3
-  static constexpr int kDecGroups = SQ_PAIR_DEC_GROUPS;  // decode groups take k-steps in turn
-  static constexpr int kDecWarps = 8 * kDecGroups;       // 8 warps per group: one 32-weight unit per thread
+  static constexpr int kDecWarps = 16;   // warps 4-19: one 32-weight unit per thread per stage
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
   static constexpr int kMmaWarp = kTmaWarp + 1;
-  static constexpr int kThreads = 32 * (kMmaWarp + 1);
-  static constexpr uint32_t kSignalBytes = 4 * 16;  // st.async bytes per stage: 8 decode warps x 2 CTAs
-  static constexpr int kStages = 6;
-  static constexpr int kA = 128 * kBK * 2;  // 16 KiB: this CTA's 128 activation rows
-  static constexpr int kB = 128 * kBK * 2;  // 16 KiB: this CTA's half of the decoded weight tile
-  static constexpr int kC = 4096;           // packed codes of that half
+  static constexpr int kGateWarp = kMmaWarp + 1;  // leader: acquires "decoded" at cluster scope for the MMA thread
+  static constexpr int kThreads = 32 * (kGateWarp + 1);
+  static constexpr int kBK = 128;        // contraction depth of a stage: 8 MMAs of K = 16
+  static constexpr int kStages = 3;
+  static constexpr int kA = 128 * kBK * 2;  // 32 KiB: this CTA's 128 activation rows, two 64-wide K chunks
+  static constexpr int kB = 128 * kBK * 2;  // 32 KiB: this CTA's half of the decoded weight tile
+  static constexpr int kC = 128 * kBK / 2;  // 8 KiB: packed codes of that half (64-byte rows, 64-byte swizzle)
   static constexpr int kStageBytes = kA + kB + kC;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 1024;
   static constexpr uint32_t kTx = kA + kC;
+  static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;  // st.async bytes per stage: all decode warps, 2 CTAs
   static constexpr int kTile = 256;         // output tile is kTile x kTile per pair
 };
 
-// Weight coordinates of decode unit u (0..255) of this CTA's half at k-step kb.
+// Decode unit u (0..511) of this CTA's half at stage kb covers 32 consecutive
+// weights: row (u & 7) + 8 * (u >> 5) of the half, quarter (u >> 3) & 3 of its
+// 128 columns (k for FWD, k-columns of the MN-major tile for DX), so the 8
+// lanes that share a shared-memory wavefront always touch 8 different rows.
 template <int MODE>
 __device__ __forceinline__ void pair_unit_coords(int u, int64_t half0, int kb, int64_t &n, int64_t &k) {
-  if (MODE == MODE_FWD) {  // 128 out-feature rows x 64 k
-    n = half0 + (u >> 1);
-    k = static_cast<int64_t>(kb) * kBK + 32 * (u & 1);
-  } else {  // 64 contraction rows x 128 k-columns
-    n = static_cast<int64_t>(kb) * kBK + (u & 7) + 8 * (u >> 5);
-    k = half0 + 32 * ((u >> 3) & 3);
+  const int row = (u & 7) + 8 * (u >> 5), quarter = (u >> 3) & 3;
+  if (MODE == MODE_FWD) {  // 128 out-feature rows x 128 k
+    n = half0 + row;
+    k = static_cast<int64_t>(kb) * PairCfg::kBK + 32 * quarter;
+  } else {  // 128 contraction rows x 128 k-columns
+    n = static_cast<int64_t>(kb) * PairCfg::kBK + row;
+    k = half0 + 32 * quarter;
   }
 }
 
@@ -653,12 +667,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint64_t *afull = bars;             // this CTA's TMA tiles landed            (1 arrival + tx)
   uint64_t *empty = bars + S;         // pair MMAs reading the stage completed   (multicast commit)
   uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded      (1 arrival + st.async tx)
-  uint64_t *tfull = bars + 3 * S;     // [2] accumulator buffer complete         (multicast commit)
+  uint64_t *gready = bars + 3 * S;    // leader: pready acquired by the gate warp (1 arrival)
+  uint64_t *tfull = bars + 4 * S;     // [2] accumulator buffer complete         (multicast commit)
   uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained      (2 x kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // [S][2][8] leader: st.async targets
+  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // [2][kDecWarps] leader: st.async targets
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -667,7 +682,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   const int nclusters = gridDim.x >> 1;
   const int total = p.tiles_m * p.tiles_n;
   const int64_t Kg = MODE == MODE_FWD ? p.K : p.N;
-  const int num_k = static_cast<int>((Kg + kBK - 1) / kBK);
+  const int num_k = static_cast<int>((Kg + C::kBK - 1) / C::kBK);
 
   auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
   auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
@@ -678,6 +693,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       mbar_init(&afull[s], 1);
       mbar_init(&empty[s], 1);
       mbar_init(&pready[s], 1);
+      mbar_init(&gready[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
@@ -713,11 +729,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
           mbar_arrive_expect_tx(&afull[s], C::kTx);
           if (rank == 0) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
-          tma_load_2d(smem_u32(stage_a(s)), &tmA, &afull[s], kb * kBK, row0);
-          if (MODE == MODE_FWD)  // codes: 128 rows x 32 bytes
-            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], kb * (kBK / 2), half0);
-          else                   // codes: 64 rows x 64 bytes, 64-byte swizzle
-            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], half0 / 2, kb * kBK);
+          // activations: two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
+          for (int j = 0; j < C::kBK / 64; ++j)
+            tma_load_2d(smem_u32(stage_a(s)) + j * 16384, &tmA, &afull[s], kb * C::kBK + 64 * j, row0);
+          if (MODE == MODE_FWD)  // codes: 128 rows x 64 bytes at (byte k/2, row n)
+            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], kb * (C::kBK / 2), half0);
+          else                   // codes: 128 contraction rows x 64 bytes
+            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], half0 / 2, kb * C::kBK);
         }
       }
       if (*abort_flag) {
@@ -727,60 +745,85 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
+    // Each tcgen05.mma blocks its thread until the tensor core takes it, so the
+    // next stage's barrier is polled between the MMAs of the current one: the
+    // tensor core then sees the next stage's MMAs right after this stage's.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
-      int it = 0, tc = 0;
-      bool ok = true;
+      // stage descriptors: stage s starts s * kStageBytes after stage 0 (start address field is >> 4).
+      // K-major tiles: K step kk lives in 64-wide chunk kk / 4 (16 KiB apart) at byte 32 * (kk % 4) of
+      // each 128-byte row; the MN-major DX tile: 16 contraction rows (2 KiB) per step, MN atoms 16 KiB apart.
+      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), 16, 1024);
+      const uint64_t bd_base = MODE == MODE_FWD ? smem_desc_sw128(smem_u32(stage_b(0)), 16, 1024)
+                                                : smem_desc_sw128(smem_u32(stage_b(0)), 16384, 1024);
+      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
+      int left = my_tiles * num_k;  // stages still to issue
+      int s = 0;                    // stage of the current k-step
+      uint32_t ph = 0;              // its phase parity
+      int tc = 0;
+      bool ok = true, ready = false;  // ready: the current stage already seen complete
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
         const int ab = tc & 1;
         const uint32_t au = static_cast<uint32_t>(tc >> 1);
         if (tc >= 2 && !(ok = mbar_wait_cluster(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
-        for (int kb = 0; kb < num_k; ++kb, ++it) {
-          const int s = it % S;
-          const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
-          if (!(ok = mbar_wait_cluster(&pready[s], ph, abort_flag, p.err))) break;  // both halves decoded
-          const uint32_t a_base = smem_u32(stage_a(s));
-          const uint32_t b_base = smem_u32(stage_b(s));
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!ready && !(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
+          const int ns = s + 1 == S ? 0 : s + 1;
+          const uint32_t nph = ns == 0 ? ph ^ 1u : ph;
+          --left;
+          ready = false;
+          const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
+          const uint64_t a0 = ad_base + so, b0 = bd_base + so;
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = smem_desc_sw128(a_base + kk * 32, 16, 1024);
-            const uint64_t bd = MODE == MODE_FWD ? smem_desc_sw128(b_base + kk * 32, 16, 1024)
-                                                 : smem_desc_sw128(b_base + kk * 2048, kBK * 128, 1024);
-            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < C::kBK / 16; ++kk) {
+            const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
+            const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
+            umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            if (left > 0 && !ready) ready = mbar_try_wait(&gready[ns], nph);
           }
           umma_commit_pair_mc(&empty[s]);
+          s = ns;
+          ph = nph;
         }
         if (ok) umma_commit_pair_mc(&tfull[ab]);
       }
       umma_commit_pair(drain);
       mbar_drain(drain, 0);
     }
+  } else if (warp == C::kGateWarp) {
+    // ------------------------------------------------------ gate (leader CTA)
+    // The cluster-scope acquire of "both halves decoded" costs a few hundred
+    // cycles even on a completed barrier; this warp pays it and hands the stage
+    // to the MMA thread through a CTA-local barrier.
+    if (lane == 0 && rank == 0) {
+      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
+      const int iters = my_tiles * num_k;
+      for (int it = 0; it < iters; ++it) {
+        const int s = it % S;
+        if (!mbar_wait_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
+        mbar_arrive(&gready[s]);
+      }
+    }
   } else if (warp >= C::kEpiWarps) {
     // ------------------------------------------------------ decode (both CTAs)
-    // Group g of 8 warps decodes the k-steps it = g, g + kDecGroups, ... of the
-    // flattened (tile, k-step) walk; every thread owns one 32-weight unit.
+    // Every decode thread turns one 32-weight unit of every stage into bf16.
     constexpr int kD = SQ_SCALE_DEPTH;
-    constexpr int kG = C::kDecGroups;
     const int dw = warp - C::kEpiWarps;
-    const int group = dw / 8;
-    const int u = (dw % 8) * 32 + lane;  // this thread's unit, 0..255
-    // walker over the flattened walk: position -> (tile, k-step)
+    const int u = dw * 32 + lane;  // this thread's unit, 0..511
     struct Pos {
       int tile, kb, tm, tn;
     };
-    auto step_by = [&](Pos &q, int n) {
-      q.kb += n;
-      while (q.kb >= num_k && q.tile < total) {
-        q.kb -= num_k;
+    auto step = [&](Pos &q) {
+      if (++q.kb == num_k) {
+        q.kb = 0;
         q.tile += nclusters;
         if (q.tile < total) tile_coords(q.tile, p.tiles_m, p.tiles_n, q.tm, q.tn);
       }
     };
     Pos cur{cluster, 0, 0, 0};
     if (cur.tile < total) tile_coords(cur.tile, p.tiles_m, p.tiles_n, cur.tm, cur.tn);
-    step_by(cur, group);
     Pos ahead = cur;
     auto scale_at = [&](const Pos &q) -> uint32_t {
       if (q.tile >= total) return 0u;
@@ -792,30 +835,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
 #pragma unroll
     for (int d = 0; d < kD; ++d) {
       sc[d] = scale_at(ahead);
-      step_by(ahead, kG);
+      step(ahead);
     }
-    // unit geometry inside the stage (fixed for the thread)
-    uint32_t c_off, b_off[4];
-    if (MODE == MODE_FWD) {
-      const int r = u >> 1, h = u & 1;
-      c_off = r * 32 + h * 16;
+    // unit geometry inside the stage (fixed for the thread): code bytes in the
+    // 64-byte-swizzled code tile, 16-byte chunks of the 128-byte-swizzled bf16 tile
+    const int row = (u & 7) + 8 * (u >> 5), quarter = (u >> 3) & 3;
+    const uint32_t c_off = row * 64 + ((quarter ^ ((row >> 1) & 3)) << 4);
+    uint32_t b_off[4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) b_off[c] = (r >> 3) * 1024 + (r & 7) * 128 + (((4 * h + c) ^ (r & 7)) << 4);
-    } else {
-      const int j = (u & 7) + 8 * (u >> 5), part = (u >> 3) & 3;
-      c_off = j * 64 + ((part ^ ((j >> 1) & 3)) << 4);
-#pragma unroll
-      for (int c = 0; c < 4; ++c)
-        b_off[c] = (part >> 1) * (kBK * 128) + j * 128 + (((4 * (part & 1) + c) ^ (j & 7)) << 4);
+    for (int c = 0; c < 4; ++c) {
+      const int chunk = 4 * (quarter & 1) + c;
+      b_off[c] = MODE == MODE_FWD
+                     ? (quarter >> 1) * 16384 + (row >> 3) * 1024 + (row & 7) * 128 + ((chunk ^ (row & 7)) << 4)
+                     : (quarter >> 1) * 16384 + row * 128 + ((chunk ^ (row & 7)) << 4);
     }
-    int it = group;
+    const uint32_t sink_addr = mapa_shared(smem_u32(&sink[rank * C::kDecWarps + dw]), 0);
+    int s = 0;
+    uint32_t ph = 0;
     bool ok = true;
     while (cur.tile < total && ok) {
 #pragma unroll
       for (int d = 0; d < kD; ++d) {
         if (cur.tile >= total || !ok) break;
-        const int s = it % S;
-        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
         if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
         ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
         __syncwarp();
@@ -842,14 +883,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
         __syncwarp();
         // tell the leader without waiting: an async store whose complete-tx on the
-        // leader's stage barrier is a cluster-scope release (both CTAs, 16 warps per stage)
-        if (lane == 0)
-          st_async_signal(mapa_shared(smem_u32(&sink[(s * 2 + rank) * 8 + dw % 8]), 0),
-                          mapa_shared(smem_u32(&pready[s]), 0));
+        // leader's stage barrier is a cluster-scope release (both CTAs, all decode warps)
+        if (lane == 0) st_async_signal(sink_addr, mapa_shared(smem_u32(&pready[s]), 0));
         sc[d] = scale_at(ahead);
-        step_by(ahead, kG);
-        step_by(cur, kG);
-        it += kG;
+        step(ahead);
+        step(cur);
+        if (++s == S) {
+          s = 0;
+          ph ^= 1u;
+        }
       }
     }
   } else {
