@@ -423,8 +423,8 @@ def run_ours(args):
         import oracle
         oracle.lib()
         host = host_copies(S, list(wl.linears))
-        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=256, n_dx=256, n_rows=4,
-                                              n_plane=1 << 17)
+        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=256, n_dx=256,
+                                              n_rows=oracle.num_threads(), n_plane=1 << 17)
         cpu = {"value": flops_step / t_full / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
                "sample": desc, "sample_seconds": round(t_spent, 2), "extrapolated_step_seconds": round(t_full, 1)}
 
@@ -482,7 +482,8 @@ def run_reference(args):
     per_step = []
     for k in range(args.warmup + args.steps):
         lin = lins[k % len(lins)]
-        t_full, t_spent, desc = oracle_sample(wl, host, [lin], n_y=64, n_dx=64, n_rows=1, n_plane=1 << 15, seed=k)
+        t_full, t_spent, desc = oracle_sample(wl, host, [lin], n_y=64, n_dx=64, n_rows=oracle.num_threads(),
+                                              n_plane=1 << 15, seed=k)
         # scale this linear's extrapolated time to the whole layer by its FLOP share
         share = 6 * wl.M * lin.N * lin.K / wl.flops()
         if k >= args.warmup:
@@ -497,8 +498,9 @@ def run_reference(args):
                    "parallelism": "host cores"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
                          "sample": "each step: one linear (cycling through the 7), 64 Y and 64 dX elements, one full "
-                                   "scale-gradient row, 32768 latents through projection and merge; full-layer time "
-                                   "extrapolated from per-element rates and the linear's FLOP share (median over steps)"},
+                                   "scale-gradient row per host thread, 32768 latents through projection and merge; "
+                                   "full-layer time extrapolated from per-element rates and the linear's FLOP share "
+                                   "(median over steps)"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)

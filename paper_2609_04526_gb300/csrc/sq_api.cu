@@ -179,8 +179,8 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
   } else {
-    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBK));  // dY, MN-major boxes 64(n) x 64(m)
-    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kBK));  // X,  MN-major boxes 64(k) x 64(m)
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));  // dY, MN-major boxes 64(n) x 96(m)
+    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kSgradBK));  // X,  MN-major boxes 64(k) x 96(m)
   }
   sqi::GemmArgs a;
   a.mode = mode;

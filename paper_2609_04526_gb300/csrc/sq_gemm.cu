@@ -352,7 +352,12 @@ struct SgradCfg {
   static constexpr int kTmaWarp = 4;
   static constexpr int kMmaWarp = 5;
   static constexpr int kThreads = 192;
-  static constexpr int kStageBytes = kAStageBytes + kBStageBytes;
+  static constexpr int kBK = kSgradBK;         // tokens per stage: 4 MMAs of K = 16
+  static constexpr int kStages = 4;
+  static constexpr int kA = kBM * kBK * 2;     // 16 KiB: dY^T tile, two MN atoms of 64 n
+  static constexpr int kB = kBN * kBK * 2;     // 32 KiB: X tile, four MN atoms of 64 k
+  static constexpr int kAtom = kBK * 128;      // bytes of one 64-wide MN atom (kBK rows of 128 B)
+  static constexpr int kStageBytes = kA + kB;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
 };
 
@@ -364,10 +369,10 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
   constexpr int B = FMT == 0 ? 16 : 32;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * C::kStageBytes);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kStages * C::kStageBytes);
   uint64_t *afull = bars;                 // TMA tiles of the stage landed      (1 arrival + tx)
-  uint64_t *empty = bars + kStages;       // MMAs reading the stage completed   (tcgen05.commit)
-  uint64_t *tfull = bars + 2 * kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
+  uint64_t *empty = bars + C::kStages;       // MMAs reading the stage completed   (tcgen05.commit)
+  uint64_t *tfull = bars + 2 * C::kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
   uint64_t *tempty = tfull + 2;           // [2] accumulator buffer drained     (kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
@@ -376,13 +381,13 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int total = p.tiles_m * p.tiles_n;
-  const int num_k = static_cast<int>((p.M + kBK - 1) / kBK);
+  const int num_k = static_cast<int>((p.M + C::kBK - 1) / C::kBK);
 
   auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
-  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + kAStageBytes; };
+  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&afull[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -414,21 +419,21 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
         tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
         const int32_t row0 = tm * kBM, col0 = tn * kBN;
         for (int kb = 0; kb < num_k; ++kb, ++it) {
-          const int s = it % kStages;
-          const uint32_t use = static_cast<uint32_t>(it / kStages);
-          if (it >= kStages && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          const int s = it % C::kStages;
+          const uint32_t use = static_cast<uint32_t>(it / C::kStages);
+          if (it >= C::kStages && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
           mbar_arrive_expect_tx(&afull[s], C::kStageBytes);
           const uint32_t a_dst = smem_u32(stage_a(s));
           const uint32_t b_dst = smem_u32(stage_b(s));
-          const int32_t kc = kb * kBK;
-          for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * (kBK * 128), &tmA, &afull[s], row0 + 64 * j, kc);
-          for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * (kBK * 128), &tmB, &afull[s], col0 + 64 * j, kc);
+          const int32_t kc = kb * C::kBK;
+          for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * C::kAtom, &tmA, &afull[s], row0 + 64 * j, kc);
+          for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * C::kAtom, &tmB, &afull[s], col0 + 64 * j, kc);
         }
       }
       if (*abort_flag) {
         // Let every issued copy land before the CTA's shared memory goes away.
-        for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
-          mbar_drain(&afull[i % kStages], static_cast<uint32_t>(i / kStages) & 1u);
+        for (int i = (it > C::kStages ? it - C::kStages : 0); i < it; ++i)
+          mbar_drain(&afull[i % C::kStages], static_cast<uint32_t>(i / C::kStages) & 1u);
       }
     }
   } else if (warp == C::kMmaWarp) {
@@ -437,8 +442,8 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
     // (each tcgen05.mma blocks until the tensor core takes it).
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, kBN, 1, 1);
-      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), kBK * 128, 1024);
-      const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), kBK * 128, 1024);
+      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), C::kAtom, 1024);
+      const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), C::kAtom, 1024);
       const int my_tiles = static_cast<int>(blockIdx.x) < total ? (total - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
       int left = my_tiles * num_k;
       int s = 0;
@@ -453,14 +458,14 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
         for (int kb = 0; kb < num_k; ++kb) {
           if (!ready && !(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
-          const int ns = s + 1 == kStages ? 0 : s + 1;
+          const int ns = s + 1 == C::kStages ? 0 : s + 1;
           const uint32_t nph = ns == 0 ? ph ^ 1u : ph;
           --left;
           ready = false;
           const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
           const uint64_t a0 = ad_base + so, b0 = bd_base + so;
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
+          for (int kk = 0; kk < C::kBK / 16; ++kk) {
             umma_bf16(d_tmem, a0 + static_cast<uint64_t>(kk * 2048 >> 4), b0 + static_cast<uint64_t>(kk * 2048 >> 4),
                       idesc, (kb > 0 || kk > 0) ? 1u : 0u);
             if (left > 0 && !ready) ready = mbar_try_wait(&afull[ns], nph);

@@ -20,6 +20,7 @@ constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
 constexpr int kStages = 4;
+constexpr int kSgradBK = 64;  // tokens per stage of the scale-gradient kernel (TMA box height)
 
 struct GemmArgs {
   int mode;

@@ -82,11 +82,11 @@ sq_status setup_current_device(NoAllocDevice **out) {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// bf16 [outer, inner] tensor in 64 x 64 boxes with the 128-byte swizzle (MN-major operand tiles).
+// bf16 [outer, inner] tensor in 64 x kSgradBK boxes with the 128-byte swizzle (MN-major operand tiles).
 bool encode_act(CUtensorMap *map, const void *ptr, int64_t inner, int64_t outer) {
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
   const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
-  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(sqi::kBK)};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(sqi::kSgradBK)};
   const cuuint32_t estr[2] = {1, 1};
   return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
