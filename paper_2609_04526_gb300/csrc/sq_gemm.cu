@@ -31,8 +31,6 @@ namespace sqi {
 namespace {
 
 constexpr uint32_t kTmemCols = 256;          // one accumulator buffer (two are allocated)
-constexpr int kAStageBytes = kBM * kBK * 2;  // 16 KiB
-constexpr int kBStageBytes = kBN * kBK * 2;  // 32 KiB
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s
 
 // ---------------------------------------------------------------- PTX helpers
@@ -438,18 +436,15 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer
-    // The next stage's barrier is polled between the MMAs of the current one
-    // (each tcgen05.mma blocks until the tensor core takes it).
+    // No barrier is polled between the MMAs of a stage: that would hold back their issue.
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, kBN, 1, 1);
       const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), C::kAtom, 1024);
       const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), C::kAtom, 1024);
-      const int my_tiles = static_cast<int>(blockIdx.x) < total ? (total - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
-      int left = my_tiles * num_k;
       int s = 0;
       uint32_t ph = 0;
       int tc = 0;
-      bool ok = true, ready = false;
+      bool ok = true;
       for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tc) {
         const int ab = tc & 1;
         const uint32_t au = static_cast<uint32_t>(tc >> 1);
@@ -457,22 +452,19 @@ __global__ void __launch_bounds__(SgradCfg::kThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!ready && !(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
-          const int ns = s + 1 == C::kStages ? 0 : s + 1;
-          const uint32_t nph = ns == 0 ? ph ^ 1u : ph;
-          --left;
-          ready = false;
+          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
           const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
           const uint64_t a0 = ad_base + so, b0 = bd_base + so;
 #pragma unroll
           for (int kk = 0; kk < C::kBK / 16; ++kk) {
             umma_bf16(d_tmem, a0 + static_cast<uint64_t>(kk * 2048 >> 4), b0 + static_cast<uint64_t>(kk * 2048 >> 4),
                       idesc, (kb > 0 || kk > 0) ? 1u : 0u);
-            if (left > 0 && !ready) ready = mbar_try_wait(&afull[ns], nph);
           }
           umma_commit(&empty[s]);
-          s = ns;
-          ph = nph;
+          if (++s == C::kStages) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (ok) umma_commit(&tfull[ab]);
       }
@@ -625,24 +617,46 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t *bar) {
                : "memory");
 }
 
+// TMA load into this CTA's shared memory whose complete-tx lands on an mbarrier
+// of either CTA of the pair (`bar_cluster` is a shared::cluster address): the
+// activation tiles of both CTAs are counted on the leader's barrier.
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster, int32_t x,
+                                                 int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+
+// Shared-memory rings of the pair kernel. The activation and decoded-weight
+// rings are released together by the MMA commit of a k-step; the code ring is
+// released by the decode warps as soon as they have read it. Because the three
+// rings advance independently, the TMA latency of the activations and the
+// decode-and-signal latency of the weights overlap instead of adding up.
 struct PairCfg {
   static constexpr int kEpiWarps = 4;    // warps 0-3
   static constexpr int kDecWarps = 16;   // warps 4-19: one 32-weight unit per thread per stage
-  static constexpr int kTmaWarp = kEpiWarps + kDecWarps;
-  static constexpr int kMmaWarp = kTmaWarp + 1;
+  static constexpr int kTmaWarp = kEpiWarps + kDecWarps;  // activation tiles
+  static constexpr int kCodeWarp = kTmaWarp + 1;          // packed-code tiles
+  static constexpr int kMmaWarp = kCodeWarp + 1;
   static constexpr int kGateWarp = kMmaWarp + 1;  // leader: acquires "decoded" at cluster scope for the MMA thread
   static constexpr int kThreads = 32 * (kGateWarp + 1);
   static constexpr int kBK = 128;        // contraction depth of a stage: 8 MMAs of K = 16
-  static constexpr int kStages = 3;
+  static constexpr int kStages = 3;      // activation and decoded-weight slots
+  static constexpr int kCStages = 4;     // code slots
   static constexpr int kA = 128 * kBK * 2;  // 32 KiB: this CTA's 128 activation rows, two 64-wide K chunks
   static constexpr int kB = 128 * kBK * 2;  // 32 KiB: this CTA's half of the decoded weight tile
   static constexpr int kC = 128 * kBK / 2;  // 8 KiB: packed codes of that half (64-byte rows, 64-byte swizzle)
-  static constexpr int kStageBytes = kA + kB + kC;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 1024;
-  static constexpr uint32_t kTx = kA + kC;
-  static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;  // st.async bytes per stage: all decode warps, 2 CTAs
+  static constexpr int kOffB = kStages * kA;
+  static constexpr int kOffC = kOffB + kStages * kB;
+  static constexpr int kOffBar = kOffC + kCStages * kC;
+  static constexpr int kSmemBytes = kOffBar + 1024 + 1024;
+  static constexpr uint32_t kATx = 2 * kA;                      // both CTAs' activation tiles, on the leader
+  static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;   // st.async bytes per stage: all decode warps, 2 CTAs
   static constexpr int kTile = 256;         // output tile is kTile x kTile per pair
 };
+static_assert(PairCfg::kSmemBytes <= 232448, "pair kernel exceeds the opt-in shared memory of one CTA");
 
 // Decode unit u (0..511) of this CTA's half at stage kb covers 32 consecutive
 // weights: row (u & 7) + 8 * (u >> 5) of the half, quarter (u >> 3) & 3 of its
@@ -666,15 +680,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
                         const KParams p) {
   using C = PairCfg;
   constexpr int S = C::kStages;
+  constexpr int SC = C::kCStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + S * C::kStageBytes);
-  uint64_t *afull = bars;             // this CTA's TMA tiles landed            (1 arrival + tx)
-  uint64_t *empty = bars + S;         // pair MMAs reading the stage completed   (multicast commit)
-  uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded      (1 arrival + st.async tx)
-  uint64_t *gready = bars + 3 * S;    // leader: pready acquired by the gate warp (1 arrival)
-  uint64_t *tfull = bars + 4 * S;     // [2] accumulator buffer complete         (multicast commit)
-  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained      (2 x kEpiWarps arrivals)
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
+  uint64_t *afull = bars;             // leader: both CTAs' activation tiles landed (1 arrival + 2 x kA tx)
+  uint64_t *empty = bars + S;         // pair MMAs reading slot s completed          (multicast commit)
+  uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded          (1 arrival + st.async tx)
+  uint64_t *gready = bars + 3 * S;    // leader: pready acquired by the gate warp     (1 arrival)
+  uint64_t *cfull = bars + 4 * S;     // [SC] this CTA's code tile landed             (1 arrival + tx)
+  uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes  (kDecWarps arrivals)
+  uint64_t *tfull = cempty + SC;      // [2] accumulator buffer complete              (multicast commit)
+  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained           (2 x kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
@@ -688,10 +705,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   const int total = p.tiles_m * p.tiles_n;
   const int64_t Kg = MODE == MODE_FWD ? p.K : p.N;
   const int num_k = static_cast<int>((Kg + C::kBK - 1) / C::kBK);
+  const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
 
-  auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
-  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
-  auto stage_c = [&](int s) { return smem + s * C::kStageBytes + C::kA + C::kB; };
+  auto ring_a = [&](int s) { return smem + s * C::kA; };
+  auto ring_b = [&](int s) { return smem + C::kOffB + s * C::kB; };
+  auto ring_c = [&](int c) { return smem + C::kOffC + c * C::kC; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -699,6 +717,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       mbar_init(&empty[s], 1);
       mbar_init(&pready[s], 1);
       mbar_init(&gready[s], 1);
+    }
+    for (int c = 0; c < SC; ++c) {
+      mbar_init(&cfull[c], 1);
+      mbar_init(&cempty[c], C::kDecWarps);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
@@ -719,7 +741,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == C::kTmaWarp) {
-    // ------------------------------------------------------ TMA producer (both CTAs)
+    // ------------------------------------------------------ activation TMA (both CTAs)
+    // Each CTA loads its own 128 rows; both loads complete on the leader's afull,
+    // which the leader arms with the bytes of the two.
     if (lane == 0) {
       int it = 0;
       bool ok = true;
@@ -727,46 +751,63 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         int tm, tn;
         tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
         const int32_t row0 = tm * C::kTile + 128 * static_cast<int32_t>(rank);
-        const int32_t half0 = tn * C::kTile + 128 * static_cast<int32_t>(rank);
         for (int kb = 0; kb < num_k; ++kb, ++it) {
           const int s = it % S;
           const uint32_t use = static_cast<uint32_t>(it / S);
           if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
-          mbar_arrive_expect_tx(&afull[s], C::kTx);
-          if (rank == 0) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
-          // activations: two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
+          if (rank == 0) mbar_arrive_expect_tx(&afull[s], C::kATx);
+          const uint32_t bar = mapa_shared(smem_u32(&afull[s]), 0);
+          // two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
           for (int j = 0; j < C::kBK / 64; ++j)
-            tma_load_2d(smem_u32(stage_a(s)) + j * 16384, &tmA, &afull[s], kb * C::kBK + 64 * j, row0);
-          if (MODE == MODE_FWD)  // codes: 128 rows x 64 bytes at (byte k/2, row n)
-            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], kb * (C::kBK / 2), half0);
-          else                   // codes: 128 contraction rows x 64 bytes
-            tma_load_2d(smem_u32(stage_c(s)), &tmC, &afull[s], half0 / 2, kb * C::kBK);
+            tma_load_2d_pair(smem_u32(ring_a(s)) + j * 16384, &tmA, bar, kb * C::kBK + 64 * j, row0);
         }
       }
-      if (*abort_flag) {
+      if (*abort_flag && rank == 0) {
         for (int i = (it > S ? it - S : 0); i < it; ++i)
           mbar_drain(&afull[i % S], static_cast<uint32_t>(i / S) & 1u);
       }
     }
+  } else if (warp == C::kCodeWarp) {
+    // ------------------------------------------------------ code TMA (both CTAs)
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        int tm, tn;
+        tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
+        const int32_t half0 = tn * C::kTile + 128 * static_cast<int32_t>(rank);
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int c = it % SC;
+          const uint32_t use = static_cast<uint32_t>(it / SC);
+          if (it >= SC && !(ok = mbar_wait(&cempty[c], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          mbar_arrive_expect_tx(&cfull[c], C::kC);
+          if (MODE == MODE_FWD)  // 128 rows x 64 bytes at (byte k/2, row n)
+            tma_load_2d(smem_u32(ring_c(c)), &tmC, &cfull[c], kb * (C::kBK / 2), half0);
+          else                   // 128 contraction rows x 64 bytes
+            tma_load_2d(smem_u32(ring_c(c)), &tmC, &cfull[c], half0 / 2, kb * C::kBK);
+        }
+      }
+      if (*abort_flag) {
+        for (int i = (it > SC ? it - SC : 0); i < it; ++i)
+          mbar_drain(&cfull[i % SC], static_cast<uint32_t>(i / SC) & 1u);
+      }
+    }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
-    // Each tcgen05.mma blocks its thread until the tensor core takes it, so the
-    // next stage's barrier is polled between the MMAs of the current one: the
-    // tensor core then sees the next stage's MMAs right after this stage's.
+    // A k-step needs its activation tiles (afull) and both decoded halves (gready).
+    // No barrier is polled between the MMAs of a step: that would hold back their issue.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
-      // stage descriptors: stage s starts s * kStageBytes after stage 0 (start address field is >> 4).
+      // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
       // K-major tiles: K step kk lives in 64-wide chunk kk / 4 (16 KiB apart) at byte 32 * (kk % 4) of
       // each 128-byte row; the MN-major DX tile: 16 contraction rows (2 KiB) per step, MN atoms 16 KiB apart.
-      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), 16, 1024);
-      const uint64_t bd_base = MODE == MODE_FWD ? smem_desc_sw128(smem_u32(stage_b(0)), 16, 1024)
-                                                : smem_desc_sw128(smem_u32(stage_b(0)), 16384, 1024);
-      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
-      int left = my_tiles * num_k;  // stages still to issue
-      int s = 0;                    // stage of the current k-step
+      const uint64_t ad_base = smem_desc_sw128(smem_u32(ring_a(0)), 16, 1024);
+      const uint64_t bd_base = MODE == MODE_FWD ? smem_desc_sw128(smem_u32(ring_b(0)), 16, 1024)
+                                                : smem_desc_sw128(smem_u32(ring_b(0)), 16384, 1024);
+      int s = 0;                    // slot of the current k-step
       uint32_t ph = 0;              // its phase parity
       int tc = 0;
-      bool ok = true, ready = false;  // ready: the current stage already seen complete
+      bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
         const int ab = tc & 1;
         const uint32_t au = static_cast<uint32_t>(tc >> 1);
@@ -774,23 +815,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!ready && !(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
-          const int ns = s + 1 == S ? 0 : s + 1;
-          const uint32_t nph = ns == 0 ? ph ^ 1u : ph;
-          --left;
-          ready = false;
-          const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
-          const uint64_t a0 = ad_base + so, b0 = bd_base + so;
+          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
+          if (!(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
+          const uint64_t a0 = ad_base + static_cast<uint64_t>(s * (C::kA >> 4));
+          const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
 #pragma unroll
           for (int kk = 0; kk < C::kBK / 16; ++kk) {
             const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
             const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
             umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
-            if (left > 0 && !ready) ready = mbar_try_wait(&gready[ns], nph);
           }
           umma_commit_pair_mc(&empty[s]);
-          s = ns;
-          ph = nph;
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (ok) umma_commit_pair_mc(&tfull[ab]);
       }
@@ -801,19 +840,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ gate (leader CTA)
     // The cluster-scope acquire of "both halves decoded" costs a few hundred
     // cycles even on a completed barrier; this warp pays it and hands the stage
-    // to the MMA thread through a CTA-local barrier.
+    // to the MMA thread through a CTA-local barrier. It also arms pready with
+    // the signal bytes of each use (decode warps may signal before it is armed:
+    // the missing arrival keeps the phase open).
     if (lane == 0 && rank == 0) {
-      const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
       const int iters = my_tiles * num_k;
+      for (int s = 0; s < S && s < iters; ++s) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
         if (!mbar_wait_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
+        if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
     }
   } else if (warp >= C::kEpiWarps) {
     // ------------------------------------------------------ decode (both CTAs)
-    // Every decode thread turns one 32-weight unit of every stage into bf16.
+    // Every decode thread turns one 32-weight unit of every stage into bf16:
+    // codes from the code ring, into the decoded slot the MMAs of k-step it - S freed.
     constexpr int kD = SQ_SCALE_DEPTH;
     const int dw = warp - C::kEpiWarps;
     const int u = dw * 32 + lane;  // this thread's unit, 0..511
@@ -855,14 +898,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
                      : (quarter >> 1) * 16384 + row * 128 + ((chunk ^ (row & 7)) << 4);
     }
     const uint32_t sink_addr = mapa_shared(smem_u32(&sink[rank * C::kDecWarps + dw]), 0);
-    int s = 0;
-    uint32_t ph = 0;
+    int it = 0, s = 0, cs = 0;
+    uint32_t ph = 0, cph = 0;  // phase parities of the decoded slot and the code slot
     bool ok = true;
     while (cur.tile < total && ok) {
 #pragma unroll
       for (int d = 0; d < kD; ++d) {
         if (cur.tile >= total || !ok) break;
-        if (lane == 0) ok = mbar_wait(&afull[s], ph, abort_flag, p.err);
+        if (lane == 0) {
+          ok = mbar_wait(&cfull[cs], cph, abort_flag, p.err);
+          if (ok && it >= S) ok = mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.err);
+        }
         ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
         __syncwarp();
         if (!ok) break;
@@ -873,8 +919,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         } else {
           sc_lo = sc_hi = scale_bf16x2<1>(sc[d]);
         }
-        const uint4 cw = lds128(smem_u32(stage_c(s)) + c_off);
-        const uint32_t b_base = smem_u32(stage_b(s));
+        const uint4 cw = lds128(smem_u32(ring_c(cs)) + c_off);
+        const uint32_t b_base = smem_u32(ring_b(s));
         const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -887,15 +933,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         }
         fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
         __syncwarp();
-        // tell the leader without waiting: an async store whose complete-tx on the
-        // leader's stage barrier is a cluster-scope release (both CTAs, all decode warps)
-        if (lane == 0) st_async_signal(sink_addr, mapa_shared(smem_u32(&pready[s]), 0));
+        if (lane == 0) {
+          mbar_arrive(&cempty[cs]);  // the warp's code reads are done
+          // tell the leader without waiting: an async store whose complete-tx on the
+          // leader's stage barrier is a cluster-scope release (both CTAs, all decode warps)
+          st_async_signal(sink_addr, mapa_shared(smem_u32(&pready[s]), 0));
+        }
         sc[d] = scale_at(ahead);
         step(ahead);
         step(cur);
+        ++it;
         if (++s == S) {
           s = 0;
           ph ^= 1u;
+        }
+        if (++cs == SC) {
+          cs = 0;
+          cph ^= 1u;
         }
       }
     }

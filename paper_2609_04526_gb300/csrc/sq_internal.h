@@ -14,13 +14,11 @@ enum GemmMode : int {
   MODE_SGRAD = 2   // g  = blockreduce(code * dY^T X)  (GEMM M=out, N=in, contraction=tokens)
 };
 
-// Tile shape of the tcgen05 contraction kernels: one 128 x 256 fp32
-// accumulator in TMEM per CTA, 64-deep k-steps through a 4-stage smem ring.
+// Tile of the scale-gradient kernel: one 128 x 256 fp32 accumulator in TMEM per
+// CTA, kSgradBK tokens per shared-memory stage (also the height of its TMA boxes).
 constexpr int kBM = 128;
 constexpr int kBN = 256;
-constexpr int kBK = 64;
-constexpr int kStages = 4;
-constexpr int kSgradBK = 64;  // tokens per stage of the scale-gradient kernel (TMA box height)
+constexpr int kSgradBK = 64;
 
 struct GemmArgs {
   int mode;
