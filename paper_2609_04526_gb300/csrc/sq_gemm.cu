@@ -687,7 +687,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint64_t *afull = bars;             // leader: both CTAs' activation tiles landed (1 arrival + 2 x kA tx)
   uint64_t *empty = bars + S;         // pair MMAs reading slot s completed          (multicast commit)
   uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded          (1 arrival + st.async tx)
-  uint64_t *gready = bars + 3 * S;    // leader: pready acquired by the gate warp     (1 arrival)
+  uint64_t *gready = bars + 3 * S;    // leader: pready and afull seen by the gate warp (1 arrival)
   uint64_t *cfull = bars + 4 * S;     // [SC] this CTA's code tile landed             (1 arrival + tx)
   uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes  (kDecWarps arrivals)
   uint64_t *tfull = cempty + SC;      // [2] accumulator buffer complete              (multicast commit)
@@ -794,8 +794,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
-    // A k-step needs its activation tiles (afull) and both decoded halves (gready).
-    // No barrier is polled between the MMAs of a step: that would hold back their issue.
+    // A k-step needs its activation tiles and both decoded halves, which the gate
+    // warp folds into one barrier (gready): every barrier wait of this thread costs
+    // issue time the tensor core cannot hide. For the same reason no barrier is
+    // polled between the MMAs of a step.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
       // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
@@ -815,7 +817,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + ab * kTmemCols;
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
           if (!(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
           const uint64_t a0 = ad_base + static_cast<uint64_t>(s * (C::kA >> 4));
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
@@ -838,17 +839,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kGateWarp) {
     // ------------------------------------------------------ gate (leader CTA)
-    // The cluster-scope acquire of "both halves decoded" costs a few hundred
-    // cycles even on a completed barrier; this warp pays it and hands the stage
-    // to the MMA thread through a CTA-local barrier. It also arms pready with
-    // the signal bytes of each use (decode warps may signal before it is armed:
-    // the missing arrival keeps the phase open).
+    // Waits, for each k-step, for both decoded halves (pready, a cluster-scope
+    // acquire that costs a few hundred cycles even on a completed barrier) and for
+    // both CTAs' activation tiles (afull), then hands the step to the MMA thread
+    // through one CTA-local barrier. It also arms pready with the signal bytes of
+    // each use (decode warps may signal before it is armed: the missing arrival
+    // keeps the phase open).
     if (lane == 0 && rank == 0) {
       const int iters = my_tiles * num_k;
       for (int s = 0; s < S && s < iters; ++s) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
-        if (!mbar_wait_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
+        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+        if (!mbar_wait_cluster(&pready[s], ph, abort_flag, p.err)) break;
+        if (!mbar_wait(&afull[s], ph, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
