@@ -90,8 +90,9 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   return SQ_OK;
 }
 
-// 2-D tensor [outer, inner] (row-major, inner contiguous) loaded in
-// box_inner x box_outer tiles; out-of-range elements read as zero.
+// 2-D tensor [outer, inner] (row-major, inner contiguous) moved in
+// box_inner x box_outer tiles; out-of-range elements read as zero and are
+// not written.
 sq_status make_map(sq_handle h, CUtensorMap *map, const void *ptr, CUtensorMapDataType dtype, int elem_bytes,
                    int64_t inner, int64_t outer, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
@@ -166,21 +167,28 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
                    void *out, const uint8_t *mask, cudaStream_t stream) {
   DeviceState *dev = nullptr;
   SQ_TRY(ensure_device(h, &dev));
-  CUtensorMap tmA, tmB;
+  CUtensorMap tmA, tmB, tmOut;
   const int64_t K2 = w->K / 2;  // code bytes per row
   if (mode == sqi::MODE_FWD) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));  // X, 128 x 64 K-major boxes
     // codes: 128 rows x 64 bytes (128 weights) per stage and CTA of the pair, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
+    // Y [M, N]: 32 x 32 store boxes (the epilogue's staging tiles), 64-byte swizzle
+    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->N, M, 32, 32,
+                    CU_TENSOR_MAP_SWIZZLE_64B));
   } else if (mode == sqi::MODE_DX) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));  // dY, 128 x 64 K-major boxes
     // codes: 128 contraction rows x 64 bytes (128 weights) per stage and CTA, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
+    // dX [M, K]: 32 x 32 store boxes, 64-byte swizzle
+    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->K, M, 32, 32,
+                    CU_TENSOR_MAP_SWIZZLE_64B));
   } else {
-    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));  // dY, MN-major boxes 64(n) x 96(m)
-    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kSgradBK));  // X,  MN-major boxes 64(k) x 96(m)
+    // dY and X as MN-major boxes of 64 features x kSgradBK tokens
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));
+    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kSgradBK));
   }
   sqi::GemmArgs a;
   a.mode = mode;
@@ -194,7 +202,7 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   a.out = out;
   a.mask = mask;
   a.err = dev->err_word;
-  cudaError_t e = sqi::launch_gemm(a, tmA, tmB, dev->sm_count, stream);
+  cudaError_t e = sqi::launch_gemm(a, tmA, tmB, mode == sqi::MODE_SGRAD ? nullptr : &tmOut, dev->sm_count, stream);
   if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
   return SQ_OK;
 }

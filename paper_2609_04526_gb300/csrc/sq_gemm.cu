@@ -617,6 +617,25 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t *bar) {
                : "memory");
 }
 
+// TMA store of one box from this CTA's shared memory, tracked by the thread's bulk groups.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+
+// Wait until at most N of this thread's bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+// Wait until all of this thread's bulk groups have completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // TMA load into this CTA's shared memory whose complete-tx lands on an mbarrier
 // of either CTA of the pair (`bar_cluster` is a shared::cluster address): the
 // activation tiles of both CTAs are counted on the leader's barrier.
@@ -629,32 +648,39 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       : "memory");
 }
 
-// Shared-memory rings of the pair kernel. The activation and decoded-weight
-// rings are released together by the MMA commit of a k-step; the code ring is
-// released by the decode warps as soon as they have read it. Because the three
-// rings advance independently, the TMA latency of the activations and the
-// decode-and-signal latency of the weights overlap instead of adding up.
+// Shared-memory rings of the pair kernel, each advancing on its own:
+//   activations     kAStages slots of 128 rows x one 128-deep stage (32 KiB): a
+//                   k-step loads two of them, one per 256-row half of the tile;
+//   decoded weights kStages slots of this CTA's 128 weight rows x one stage (32 KiB);
+//   packed codes    kCStages slots (8 KiB), released by the decode warps once read;
+//   output staging  two 2 KiB boxes per epilogue warp for the TMA stores of the result.
+// A pair computes a 512 x 256 output tile: every decoded weight stage feeds the
+// MMAs of both 256-row halves, into two TMEM accumulators (all 512 columns), so
+// the decode-and-signal chain of a stage is covered by twice the tensor work.
 struct PairCfg {
   static constexpr int kEpiWarps = 4;    // warps 0-3
   static constexpr int kDecWarps = 16;   // warps 4-19: one 32-weight unit per thread per stage
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;  // activation tiles
   static constexpr int kCodeWarp = kTmaWarp + 1;          // packed-code tiles
   static constexpr int kMmaWarp = kCodeWarp + 1;
-  static constexpr int kGateWarp = kMmaWarp + 1;  // leader: acquires "decoded" at cluster scope for the MMA thread
+  static constexpr int kGateWarp = kMmaWarp + 1;  // leader: folds "decoded" and "activations landed" into one barrier
   static constexpr int kThreads = 32 * (kGateWarp + 1);
-  static constexpr int kBK = 128;        // contraction depth of a stage: 8 MMAs of K = 16
-  static constexpr int kStages = 3;      // activation and decoded-weight slots
-  static constexpr int kCStages = 4;     // code slots
-  static constexpr int kA = 128 * kBK * 2;  // 32 KiB: this CTA's 128 activation rows, two 64-wide K chunks
+  static constexpr int kBK = 128;        // contraction depth of a stage: 8 MMAs of K = 16 per tile half
+  static constexpr int kAStages = 4;     // activation slots (two per k-step)
+  static constexpr int kStages = 2;      // decoded-weight slots (a k-step feeds 16 MMAs)
+  static constexpr int kCStages = 2;     // code slots (a k-step lasts >= 2048 tensor cycles)
+  static constexpr int kA = 128 * kBK * 2;  // 32 KiB: this CTA's 128 rows of one tile half, two 64-wide K chunks
   static constexpr int kB = 128 * kBK * 2;  // 32 KiB: this CTA's half of the decoded weight tile
   static constexpr int kC = 128 * kBK / 2;  // 8 KiB: packed codes of that half (64-byte rows, 64-byte swizzle)
-  static constexpr int kOffB = kStages * kA;
+  static constexpr int kOffB = kAStages * kA;
   static constexpr int kOffC = kOffB + kStages * kB;
-  static constexpr int kOffBar = kOffC + kCStages * kC;
+  static constexpr int kOffS = kOffC + kCStages * kC;   // output staging: [kEpiWarps][2][32 x 32 bf16]
+  static constexpr int kOffBar = kOffS + kEpiWarps * 2 * 2048;
   static constexpr int kSmemBytes = kOffBar + 1024 + 1024;
   static constexpr uint32_t kATx = 2 * kA;                      // both CTAs' activation tiles, on the leader
   static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;   // st.async bytes per stage: all decode warps, 2 CTAs
-  static constexpr int kTile = 256;         // output tile is kTile x kTile per pair
+  static constexpr int kTile = 256;         // output columns of a pair tile (and rows of one half)
+  static constexpr int kMTile = 512;        // output rows of a pair tile: two halves of kTile
 };
 static_assert(PairCfg::kSmemBytes <= 232448, "pair kernel exceeds the opt-in shared memory of one CTA");
 
@@ -677,21 +703,23 @@ __device__ __forceinline__ void pair_unit_coords(int u, int64_t half0, int kb, i
 template <int MODE, int FMT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1)
     sq_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmC,
-                        const KParams p) {
+                        const __grid_constant__ CUtensorMap tmO, const KParams p) {
   using C = PairCfg;
+  constexpr int SA = C::kAStages;
   constexpr int S = C::kStages;
   constexpr int SC = C::kCStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
-  uint64_t *afull = bars;             // leader: both CTAs' activation tiles landed (1 arrival + 2 x kA tx)
-  uint64_t *empty = bars + S;         // pair MMAs reading slot s completed          (multicast commit)
-  uint64_t *pready = bars + 2 * S;    // leader: both weight halves decoded          (1 arrival + st.async tx)
-  uint64_t *gready = bars + 3 * S;    // leader: pready and afull seen by the gate warp (1 arrival)
-  uint64_t *cfull = bars + 4 * S;     // [SC] this CTA's code tile landed             (1 arrival + tx)
-  uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes  (kDecWarps arrivals)
-  uint64_t *tfull = cempty + SC;      // [2] accumulator buffer complete              (multicast commit)
-  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained           (2 x kEpiWarps arrivals)
+  uint64_t *afull = bars;             // [SA] leader: both CTAs' activation tiles landed (1 arrival + 2 x kA tx)
+  uint64_t *aempty = afull + SA;      // [SA] pair MMAs reading activation slot a done   (multicast commit)
+  uint64_t *empty = aempty + SA;      // [S] pair MMAs reading decoded slot s done       (multicast commit)
+  uint64_t *pready = empty + S;       // [S] leader: both weight halves decoded          (1 arrival + st.async tx)
+  uint64_t *gready = pready + S;      // [S] leader: pready and both afull seen by the gate (1 arrival)
+  uint64_t *cfull = gready + S;       // [SC] this CTA's code tile landed                 (1 arrival + tx)
+  uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes      (kDecWarps arrivals)
+  uint64_t *tfull = cempty + SC;      // both accumulators of the tile complete           (multicast commit)
+  uint64_t *tempty = tfull + 1;       // [2] leader: both epilogues drained accumulator h (2 x kEpiWarps arrivals)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
@@ -707,13 +735,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   const int num_k = static_cast<int>((Kg + C::kBK - 1) / C::kBK);
   const int my_tiles = cluster < total ? (total - cluster + nclusters - 1) / nclusters : 0;
 
-  auto ring_a = [&](int s) { return smem + s * C::kA; };
+  auto ring_a = [&](int a) { return smem + a * C::kA; };
   auto ring_b = [&](int s) { return smem + C::kOffB + s * C::kB; };
   auto ring_c = [&](int c) { return smem + C::kOffC + c * C::kC; };
 
   if (threadIdx.x == 0) {
+    for (int a = 0; a < SA; ++a) {
+      mbar_init(&afull[a], 1);
+      mbar_init(&aempty[a], 1);
+    }
     for (int s = 0; s < S; ++s) {
-      mbar_init(&afull[s], 1);
       mbar_init(&empty[s], 1);
       mbar_init(&pready[s], 1);
       mbar_init(&gready[s], 1);
@@ -722,10 +753,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       mbar_init(&cfull[c], 1);
       mbar_init(&cempty[c], C::kDecWarps);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 2 * C::kEpiWarps);
-    }
+    mbar_init(tfull, 1);
+    for (int h = 0; h < 2; ++h) mbar_init(&tempty[h], 2 * C::kEpiWarps);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -734,6 +763,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   if (warp == C::kTmaWarp && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmC);
+    tma_prefetch_desc(&tmO);
   }
   tc_fence_before();
   cluster_sync_all();
@@ -742,29 +772,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
 
   if (warp == C::kTmaWarp) {
     // ------------------------------------------------------ activation TMA (both CTAs)
-    // Each CTA loads its own 128 rows; both loads complete on the leader's afull,
-    // which the leader arms with the bytes of the two.
+    // Per k-step, one slot per tile half: each CTA loads its own 128 rows of the
+    // half; both loads complete on the leader's afull, which the leader arms with
+    // the bytes of the two.
     if (lane == 0) {
-      int it = 0;
+      int ja = 0;  // activation slots filled
       bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters) {
         int tm, tn;
         tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-        const int32_t row0 = tm * C::kTile + 128 * static_cast<int32_t>(rank);
-        for (int kb = 0; kb < num_k; ++kb, ++it) {
-          const int s = it % S;
-          const uint32_t use = static_cast<uint32_t>(it / S);
-          if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
-          if (rank == 0) mbar_arrive_expect_tx(&afull[s], C::kATx);
-          const uint32_t bar = mapa_shared(smem_u32(&afull[s]), 0);
-          // two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
-          for (int j = 0; j < C::kBK / 64; ++j)
-            tma_load_2d_pair(smem_u32(ring_a(s)) + j * 16384, &tmA, bar, kb * C::kBK + 64 * j, row0);
+        const int32_t row0 = tm * C::kMTile + 128 * static_cast<int32_t>(rank);
+        for (int kb = 0; kb < num_k && ok; ++kb) {
+          for (int h = 0; h < 2; ++h, ++ja) {
+            const int a = ja % SA;
+            const uint32_t use = static_cast<uint32_t>(ja / SA);
+            if (ja >= SA && !(ok = mbar_wait(&aempty[a], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+            if (rank == 0) mbar_arrive_expect_tx(&afull[a], C::kATx);
+            const uint32_t bar = mapa_shared(smem_u32(&afull[a]), 0);
+            // two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
+            for (int j = 0; j < C::kBK / 64; ++j)
+              tma_load_2d_pair(smem_u32(ring_a(a)) + j * 16384, &tmA, bar, kb * C::kBK + 64 * j, row0 + C::kTile * h);
+          }
         }
       }
       if (*abort_flag && rank == 0) {
-        for (int i = (it > S ? it - S : 0); i < it; ++i)
-          mbar_drain(&afull[i % S], static_cast<uint32_t>(i / S) & 1u);
+        for (int i = (ja > SA ? ja - SA : 0); i < ja; ++i)
+          mbar_drain(&afull[i % SA], static_cast<uint32_t>(i / SA) & 1u);
       }
     }
   } else if (warp == C::kCodeWarp) {
@@ -794,10 +827,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
-    // A k-step needs its activation tiles and both decoded halves, which the gate
-    // warp folds into one barrier (gready): every barrier wait of this thread costs
-    // issue time the tensor core cannot hide. For the same reason no barrier is
-    // polled between the MMAs of a step.
+    // A k-step needs the activation tiles of both halves and both decoded weight
+    // halves, which the gate warp folds into one barrier (gready): every barrier
+    // wait of this thread costs issue time the tensor core cannot hide. For the
+    // same reason no barrier is polled between MMAs.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
       // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
@@ -806,33 +839,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       const uint64_t ad_base = smem_desc_sw128(smem_u32(ring_a(0)), 16, 1024);
       const uint64_t bd_base = MODE == MODE_FWD ? smem_desc_sw128(smem_u32(ring_b(0)), 16, 1024)
                                                 : smem_desc_sw128(smem_u32(ring_b(0)), 16384, 1024);
-      int s = 0;                    // slot of the current k-step
-      uint32_t ph = 0;              // its phase parity
+      int s = 0, a = 0;             // decoded slot of the current k-step, activation slot of its first half
+      uint32_t ph = 0;              // phase parity of the decoded slot
       int tc = 0;
       bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
-        const int ab = tc & 1;
-        const uint32_t au = static_cast<uint32_t>(tc >> 1);
-        if (tc >= 2 && !(ok = mbar_wait_cluster(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + ab * kTmemCols;
         for (int kb = 0; kb < num_k; ++kb) {
           if (!(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
-          const uint64_t a0 = ad_base + static_cast<uint64_t>(s * (C::kA >> 4));
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
 #pragma unroll
-          for (int kk = 0; kk < C::kBK / 16; ++kk) {
-            const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
-            const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
-            umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          for (int h = 0; h < 2; ++h) {
+            // the previous tile's epilogue has drained accumulator h
+            if (kb == 0 && tc >= 1 &&
+                !(ok = mbar_wait_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
+              break;
+            if (kb == 0) tc_fence_after();
+            const uint32_t d_tmem = tmem_base + h * kTmemCols;
+            const uint64_t a0 = ad_base + static_cast<uint64_t>(a * (C::kA >> 4));
+#pragma unroll
+            for (int kk = 0; kk < C::kBK / 16; ++kk) {
+              const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
+              const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
+              umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            }
+            umma_commit_pair_mc(&aempty[a]);
+            if (++a == SA) a = 0;
           }
+          if (!ok) break;
           umma_commit_pair_mc(&empty[s]);
           if (++s == S) {
             s = 0;
             ph ^= 1u;
           }
         }
-        if (ok) umma_commit_pair_mc(&tfull[ab]);
+        if (ok) umma_commit_pair_mc(tfull);
       }
       umma_commit_pair(drain);
       mbar_drain(drain, 0);
@@ -841,18 +881,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ gate (leader CTA)
     // Waits, for each k-step, for both decoded halves (pready, a cluster-scope
     // acquire that costs a few hundred cycles even on a completed barrier) and for
-    // both CTAs' activation tiles (afull), then hands the step to the MMA thread
-    // through one CTA-local barrier. It also arms pready with the signal bytes of
-    // each use (decode warps may signal before it is armed: the missing arrival
-    // keeps the phase open).
+    // the activation tiles of both tile halves (afull), then hands the step to the
+    // MMA thread through one CTA-local barrier. It also arms pready with the signal
+    // bytes of each use (decode warps may signal before it is armed: the missing
+    // arrival keeps the phase open).
     if (lane == 0 && rank == 0) {
       const int iters = my_tiles * num_k;
       for (int s = 0; s < S && s < iters; ++s) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
-        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
-        if (!mbar_wait_cluster(&pready[s], ph, abort_flag, p.err)) break;
-        if (!mbar_wait(&afull[s], ph, abort_flag, p.err)) break;
+        if (!mbar_wait_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
+        bool ok = true;
+        for (int h = 0; h < 2 && ok; ++h) {
+          const int ja = 2 * it + h;
+          ok = mbar_wait(&afull[ja % SA], static_cast<uint32_t>(ja / SA) & 1u, abort_flag, p.err);
+        }
+        if (!ok) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
@@ -959,45 +1003,59 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else {
     // ------------------------------------------------------ epilogue (warps 0-3, both CTAs)
-    const int r = warp * 32 + lane;
+    // Drains accumulator 0 (rows 0-255 of the tile), releases it so the next
+    // tile's first MMAs can start, then drains accumulator 1. Each warp turns its
+    // 32 TMEM lanes x 32 columns into a bf16 box in shared memory (64-byte
+    // swizzle, two boxes in flight) and stores it with TMA, which writes whole
+    // row segments and clips the ragged edges of the output.
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
     const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
     const float scale = FMT == 0 ? p.ws2 : 1.0f;
-    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(p.out);
+    const uint32_t stage0 = smem_u32(smem + C::kOffS + warp * 2 * 2048);
+    uint32_t row_off[4];  // this lane's 16-byte chunks of its 64-byte box row
+#pragma unroll
+    for (int q = 0; q < 4; ++q) row_off[q] = lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4);
+    int nb = 0;  // boxes stored by this warp
     int tc = 0;
     for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
       int tm, tn;
       tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
-      const int64_t grow = static_cast<int64_t>(tm) * C::kTile + 128 * rank + r;
-      const int64_t col0 = static_cast<int64_t>(tn) * C::kTile;
-      const int ab = tc & 1;
-      const uint32_t au = static_cast<uint32_t>(tc >> 1);
-      if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
+      const int32_t col0 = tn * C::kTile;
+      if (!mbar_wait(tfull, static_cast<uint32_t>(tc) & 1u, abort_flag, p.err)) break;
       tc_fence_after();
-      const uint32_t t_buf = t_row + ab * kTmemCols;
-      for (int c0 = 0; c0 < C::kTile; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(t_buf + c0, v);
-        tmem_ld_wait();
-        if (grow >= p.M) continue;
+      for (int h = 0; h < 2; ++h) {
+        const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * warp;
+        const uint32_t t_buf = t_row + h * kTmemCols;
+        for (int c0 = 0; c0 < C::kTile; c0 += 32, ++nb) {
+          uint32_t v[32];
+          tmem_ld32(t_buf + c0, v);
+          tmem_ld_wait();
+          uint32_t packed[16];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int64_t gc = col0 + c0 + 8 * q;
-          if (gc >= Ng) continue;
-          uint32_t packed[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v[8 * q + 2 * e]) * scale,
-                                                            __uint_as_float(v[8 * q + 2 * e + 1]) * scale);
+          for (int e = 0; e < 16; ++e) {
+            const __nv_bfloat162 h2 =
+                __floats2bfloat162_rn(__uint_as_float(v[2 * e]) * scale, __uint_as_float(v[2 * e + 1]) * scale);
             packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
           }
-          *reinterpret_cast<uint4 *>(out + grow * Ng + gc) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+          const uint32_t buf = stage0 + (nb & 1) * 2048;
+          if (lane == 0) bulk_wait_read<1>();  // the store that read this buffer two boxes ago is done with it
+          __syncwarp();
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            st_shared_v4(buf + row_off[q], packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+          fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
+          __syncwarp();
+          if (lane == 0) {
+            if (row < p.M && col0 + c0 < Ng) tma_store_2d(&tmO, buf, col0 + c0, row);
+            bulk_commit_group();
+          }
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[h]), 0));
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[ab]), 0));
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   __syncwarp();
@@ -1010,8 +1068,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
 }
 
 template <int MODE, int FMT>
-cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmC, int sm_count,
-                        cudaStream_t stream) {
+cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmC, const CUtensorMap *tmOut,
+                        int sm_count, cudaStream_t stream) {
   using C = PairCfg;
   static int attr_done_mask = 0;
   static int max_clusters[32] = {0};
@@ -1035,10 +1093,10 @@ cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
   }
   const int64_t Ng = MODE == MODE_FWD ? a.N : a.K;
   KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err,
-            static_cast<int>((a.M + C::kTile - 1) / C::kTile), static_cast<int>((Ng + C::kTile - 1) / C::kTile)};
+            static_cast<int>((a.M + C::kMTile - 1) / C::kMTile), static_cast<int>((Ng + C::kTile - 1) / C::kTile)};
   const int64_t total = static_cast<int64_t>(p.tiles_m) * p.tiles_n;
   const int64_t nc = total < max_clusters[dev & 31] ? total : max_clusters[dev & 31];
-  kernel<<<static_cast<unsigned>(2 * nc), C::kThreads, C::kSmemBytes, stream>>>(tmA, tmC, p);
+  kernel<<<static_cast<unsigned>(2 * nc), C::kThreads, C::kSmemBytes, stream>>>(tmA, tmC, *tmOut, p);
   return cudaGetLastError();
 }
 
@@ -1065,15 +1123,16 @@ cudaError_t launch_sgrad(const GemmArgs &a, const CUtensorMap &tmA, const CUtens
 
 }  // namespace
 
-cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
-                        cudaStream_t stream) {
+cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap *tmOut,
+                        int sm_count, cudaStream_t stream) {
+  if (a.mode != MODE_SGRAD && !tmOut) return cudaErrorInvalidValue;
   if (a.fmt == 0) {
-    if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 0>(a, tmA, tmB, sm_count, stream);
-    if (a.mode == MODE_DX) return launch_pair<MODE_DX, 0>(a, tmA, tmB, sm_count, stream);
+    if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 0>(a, tmA, tmB, tmOut, sm_count, stream);
+    if (a.mode == MODE_DX) return launch_pair<MODE_DX, 0>(a, tmA, tmB, tmOut, sm_count, stream);
     return launch_sgrad<0>(a, tmA, tmB, sm_count, stream);
   }
-  if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 1>(a, tmA, tmB, sm_count, stream);
-  if (a.mode == MODE_DX) return launch_pair<MODE_DX, 1>(a, tmA, tmB, sm_count, stream);
+  if (a.mode == MODE_FWD) return launch_pair<MODE_FWD, 1>(a, tmA, tmB, tmOut, sm_count, stream);
+  if (a.mode == MODE_DX) return launch_pair<MODE_DX, 1>(a, tmA, tmB, tmOut, sm_count, stream);
   return launch_sgrad<1>(a, tmA, tmB, sm_count, stream);
 }
 

@@ -32,10 +32,12 @@ struct GemmArgs {
   int *err;              // device error word
 };
 
-// Launch one contraction. tmA / tmB are the TMA descriptors of the streamed
-// bf16 operands (tmB is used by MODE_SGRAD only).
-cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
-                        cudaStream_t stream);
+// Launch one contraction. tmA is the TMA descriptor of the streamed bf16
+// activations; tmB that of the packed codes (MODE_FWD / MODE_DX) or of the second
+// bf16 operand (MODE_SGRAD); tmOut that of the bf16 output (MODE_FWD / MODE_DX:
+// 32 x 32 boxes, 64-byte swizzle; null for MODE_SGRAD).
+cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap *tmOut,
+                        int sm_count, cudaStream_t stream);
 
 cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *latent, uint8_t *bytes_out,
                            uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream);

@@ -135,7 +135,7 @@ extern "C" sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X
     a.out = g;
     a.mask = mask;
     a.err = dev->scratch;
-    if (sqi::launch_gemm(a, tmA, tmB, dev->sm_count, s) != cudaSuccess) return SQ_ERR_CUDA;
+    if (sqi::launch_gemm(a, tmA, tmB, nullptr, dev->sm_count, s) != cudaSuccess) return SQ_ERR_CUDA;
   }
   if (device_status &&
       cudaMemcpyAsync(device_status, dev->scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)

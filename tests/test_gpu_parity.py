@@ -26,7 +26,7 @@ def h():
 
 
 SMALL = [
-    # key, fmt, M, N, K      (tiles are 128 x 256 with 64-deep k-steps)
+    # key, fmt, M, N, K      (pair tiles: 512 x 256 with 128-deep k-steps; scale-gradient tiles: 128 x 256)
     ("c1", NV, 64, 256, 512),
     ("nv_ragged", NV, 300, 392, 608),
     ("mx_ragged", MX, 257, 264, 544),
