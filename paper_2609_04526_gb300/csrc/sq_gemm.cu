@@ -718,12 +718,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint64_t *gready = pready + S;      // [S] leader: pready and both afull seen by the gate (1 arrival)
   uint64_t *cfull = gready + S;       // [SC] this CTA's code tile landed                 (1 arrival + tx)
   uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes      (kDecWarps arrivals)
-  uint64_t *tfull = cempty + SC;      // both accumulators of the tile complete           (multicast commit)
-  uint64_t *tempty = tfull + 1;       // [2] leader: both epilogues drained accumulator h (2 x kEpiWarps arrivals)
+  uint64_t *tfull = cempty + SC;      // [2] accumulator h of the tile complete          (multicast commit)
+  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained accumulator h
+                                      //     (kEpiWarps arrivals + the peer warps' st.async tx)
   uint64_t *drain = tempty + 2;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // [2][kDecWarps] leader: st.async targets
+  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // leader: st.async targets, [2][kDecWarps] + [kEpiWarps]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -753,8 +754,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       mbar_init(&cfull[c], 1);
       mbar_init(&cempty[c], C::kDecWarps);
     }
-    mbar_init(tfull, 1);
-    for (int h = 0; h < 2; ++h) mbar_init(&tempty[h], 2 * C::kEpiWarps);
+    for (int h = 0; h < 2; ++h) {
+      mbar_init(&tfull[h], 1);
+      mbar_init(&tempty[h], C::kEpiWarps);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -863,6 +866,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
               umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
             }
             umma_commit_pair_mc(&aempty[a]);
+            if (kb == num_k - 1) umma_commit_pair_mc(&tfull[h]);  // the epilogue may start on accumulator h
             if (++a == SA) a = 0;
           }
           if (!ok) break;
@@ -872,7 +876,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
             ph ^= 1u;
           }
         }
-        if (ok) umma_commit_pair_mc(tfull);
       }
       umma_commit_pair(drain);
       mbar_drain(drain, 0);
@@ -1021,9 +1024,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       int tm, tn;
       tile_coords(tile, p.tiles_m, p.tiles_n, tm, tn);
       const int32_t col0 = tn * C::kTile;
-      if (!mbar_wait(tfull, static_cast<uint32_t>(tc) & 1u, abort_flag, p.err)) break;
-      tc_fence_after();
-      for (int h = 0; h < 2; ++h) {
+      bool ok = true;
+      for (int h = 0; h < 2 && ok; ++h) {
+        if (!(ok = mbar_wait(&tfull[h], static_cast<uint32_t>(tc) & 1u, abort_flag, p.err))) break;
+        tc_fence_after();
         const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * warp;
         const uint32_t t_buf = t_row + h * kTmemCols;
         for (int c0 = 0; c0 < C::kTile; c0 += 32, ++nb) {
@@ -1052,8 +1056,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[h]), 0));
+        // accumulator h drained: the leader's warps arrive (warp 0 arming the peer's
+        // bytes), the peer's warps signal with a non-blocking async store
+        if (lane == 0) {
+          if (rank == 0) {
+            if (warp == 0)
+              mbar_arrive_expect_tx(&tempty[h], 4 * C::kEpiWarps);
+            else
+              mbar_arrive(&tempty[h]);
+          } else {
+            st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
+                            mapa_shared(smem_u32(&tempty[h]), 0));
+          }
+        }
       }
+      if (!ok) break;
     }
     if (lane == 0) bulk_wait_all();
   }
