@@ -174,17 +174,17 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
     // codes: 128 rows x 64 bytes (128 weights) per stage and CTA of the pair, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
-    // Y [M, N]: 32 x 32 store boxes (the epilogue's staging tiles), 64-byte swizzle
-    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->N, M, 32, 32,
-                    CU_TENSOR_MAP_SWIZZLE_64B));
+    // Y [M, N]: 32-row x 64-column store boxes (the epilogue's staging tiles), 128-byte swizzle
+    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->N, M, 64, 32,
+                    CU_TENSOR_MAP_SWIZZLE_128B));
   } else if (mode == sqi::MODE_DX) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));  // dY, 128 x 64 K-major boxes
     // codes: 128 contraction rows x 64 bytes (128 weights) per stage and CTA, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
-    // dX [M, K]: 32 x 32 store boxes, 64-byte swizzle
-    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->K, M, 32, 32,
-                    CU_TENSOR_MAP_SWIZZLE_64B));
+    // dX [M, K]: 32-row x 64-column store boxes, 128-byte swizzle
+    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->K, M, 64, 32,
+                    CU_TENSOR_MAP_SWIZZLE_128B));
   } else {
     // dY and X as MN-major boxes of 64 features x kSgradBK tokens
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));

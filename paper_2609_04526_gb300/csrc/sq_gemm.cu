@@ -576,9 +576,6 @@ __device__ __forceinline__ void st_async_signal(uint32_t cluster_dst, uint32_t c
                : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
-}
 
 
 // TMEM allocation for a CTA pair: one warp of each CTA executes these collectively.
@@ -653,7 +650,7 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
 //                   k-step loads two of them, one per 256-row half of the tile;
 //   decoded weights kStages slots of this CTA's 128 weight rows x one stage (32 KiB);
 //   packed codes    kCStages slots (8 KiB), released by the decode warps once read;
-//   output staging  two 2 KiB boxes per epilogue warp for the TMA stores of the result.
+//   output staging  one 4 KiB box per epilogue warp for the TMA stores of the result.
 // A pair computes a 512 x 256 output tile: every decoded weight stage feeds the
 // MMAs of both 256-row halves, into two TMEM accumulators (all 512 columns), so
 // the decode-and-signal chain of a stage is covered by twice the tensor work.
@@ -674,8 +671,8 @@ struct PairCfg {
   static constexpr int kC = 128 * kBK / 2;  // 8 KiB: packed codes of that half (64-byte rows, 64-byte swizzle)
   static constexpr int kOffB = kAStages * kA;
   static constexpr int kOffC = kOffB + kStages * kB;
-  static constexpr int kOffS = kOffC + kCStages * kC;   // output staging: [kEpiWarps][2][32 x 32 bf16]
-  static constexpr int kOffBar = kOffS + kEpiWarps * 2 * 2048;
+  static constexpr int kOffS = kOffC + kCStages * kC;   // output staging: [kEpiWarps][32 x 64 bf16]
+  static constexpr int kOffBar = kOffS + kEpiWarps * 4096;
   static constexpr int kSmemBytes = kOffBar + 1024 + 1024;
   static constexpr uint32_t kATx = 2 * kA;                      // both CTAs' activation tiles, on the leader
   static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;   // st.async bytes per stage: all decode warps, 2 CTAs
@@ -1008,17 +1005,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ epilogue (warps 0-3, both CTAs)
     // Drains accumulator 0 (rows 0-255 of the tile), releases it so the next
     // tile's first MMAs can start, then drains accumulator 1. Each warp turns its
-    // 32 TMEM lanes x 32 columns into a bf16 box in shared memory (64-byte
-    // swizzle, two boxes in flight) and stores it with TMA, which writes whole
-    // row segments and clips the ragged edges of the output.
+    // 32 TMEM lanes x 64 columns into a bf16 box in shared memory (128-byte
+    // swizzle) and stores it with TMA, which writes whole 128-byte row segments
+    // and clips the ragged edges of the output.
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
     const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
     const float scale = FMT == 0 ? p.ws2 : 1.0f;
-    const uint32_t stage0 = smem_u32(smem + C::kOffS + warp * 2 * 2048);
-    uint32_t row_off[4];  // this lane's 16-byte chunks of its 64-byte box row
-#pragma unroll
-    for (int q = 0; q < 4; ++q) row_off[q] = lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4);
-    int nb = 0;  // boxes stored by this warp
+    const uint32_t box = smem_u32(smem + C::kOffS + warp * 4096);
+    const uint32_t row_base = box + lane * 128;  // this lane's 128-byte box row
     int tc = 0;
     for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
       int tm, tn;
@@ -1030,27 +1024,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         tc_fence_after();
         const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * warp;
         const uint32_t t_buf = t_row + h * kTmemCols;
-        for (int c0 = 0; c0 < C::kTile; c0 += 32, ++nb) {
-          uint32_t v[32];
-          tmem_ld32(t_buf + c0, v);
-          tmem_ld_wait();
-          uint32_t packed[16];
+        for (int c0 = 0; c0 < C::kTile; c0 += 64) {
+#pragma unroll 1
+          for (int half = 0; half < 2; ++half) {
+            uint32_t v[32];
+            tmem_ld32(t_buf + c0 + 32 * half, v);
+            tmem_ld_wait();
+            uint32_t packed[16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const __nv_bfloat162 h2 =
-                __floats2bfloat162_rn(__uint_as_float(v[2 * e]) * scale, __uint_as_float(v[2 * e + 1]) * scale);
-            packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
+            for (int e = 0; e < 16; ++e) {
+              const __nv_bfloat162 h2 =
+                  __floats2bfloat162_rn(__uint_as_float(v[2 * e]) * scale, __uint_as_float(v[2 * e + 1]) * scale);
+              packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
+            }
+            if (half == 0) {
+              if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
+              __syncwarp();
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int chunk = 4 * half + q;
+              st_shared_v4(row_base + ((chunk ^ (lane & 7)) << 4), packed[4 * q], packed[4 * q + 1],
+                           packed[4 * q + 2], packed[4 * q + 3]);
+            }
           }
-          const uint32_t buf = stage0 + (nb & 1) * 2048;
-          if (lane == 0) bulk_wait_read<1>();  // the store that read this buffer two boxes ago is done with it
-          __syncwarp();
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            st_shared_v4(buf + row_off[q], packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
           fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
           __syncwarp();
           if (lane == 0) {
-            if (row < p.M && col0 + c0 < Ng) tma_store_2d(&tmO, buf, col0 + c0, row);
+            if (row < p.M && col0 + c0 < Ng) tma_store_2d(&tmO, box, col0 + c0, row);
             bulk_commit_group();
           }
         }

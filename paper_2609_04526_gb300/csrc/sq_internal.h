@@ -35,7 +35,7 @@ struct GemmArgs {
 // Launch one contraction. tmA is the TMA descriptor of the streamed bf16
 // activations; tmB that of the packed codes (MODE_FWD / MODE_DX) or of the second
 // bf16 operand (MODE_SGRAD); tmOut that of the bf16 output (MODE_FWD / MODE_DX:
-// 32 x 32 boxes, 64-byte swizzle; null for MODE_SGRAD).
+// 32-row x 64-column boxes, 128-byte swizzle; null for MODE_SGRAD).
 cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap *tmOut,
                         int sm_count, cudaStream_t stream);
 
