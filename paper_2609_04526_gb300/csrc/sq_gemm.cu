@@ -92,6 +92,58 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
   return mbar_wait_slow(bar, parity, abort_flag, err);
 }
 
+// Non-suspending variants for the threads on the critical path of the pair
+// kernel (MMA issue, gate): mbarrier.try_wait may suspend the thread, and a
+// suspended thread resumes a few hundred cycles after the phase completes;
+// test_wait returns at once, so these spin (with the same time limit).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_test_wait_cluster(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+template <bool CLUSTER>
+__device__ __noinline__ bool mbar_spin_slow(uint64_t *bar, uint32_t parity, volatile int *abort_flag, int *err) {
+  const unsigned long long t0 = globaltimer();
+  while (true) {
+    for (int i = 0; i < 256; ++i)
+      if (CLUSTER ? mbar_test_wait_cluster(bar, parity) : mbar_test_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      atomicOr(err, kErrWaitTimeout);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ bool mbar_spin(uint64_t *bar, uint32_t parity, volatile int *abort_flag, int *err) {
+  return mbar_test_wait(bar, parity) || mbar_spin_slow<false>(bar, parity, abort_flag, err);
+}
+
+__device__ __forceinline__ bool mbar_spin_cluster(uint64_t *bar, uint32_t parity, volatile int *abort_flag,
+                                                  int *err) {
+  return mbar_test_wait_cluster(bar, parity) || mbar_spin_slow<true>(bar, parity, abort_flag, err);
+}
+
 // Bounded wait used only while tearing down after an abort: waits for work this
 // CTA already put in flight (TMA copies, MMAs), ignoring the abort flag.
 __device__ __noinline__ void mbar_drain(uint64_t *bar, uint32_t parity) {
@@ -845,13 +897,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
         for (int kb = 0; kb < num_k; ++kb) {
-          if (!(ok = mbar_wait(&gready[s], ph, abort_flag, p.err))) break;
+          if (!(ok = mbar_spin(&gready[s], ph, abort_flag, p.err))) break;
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             // the previous tile's epilogue has drained accumulator h
             if (kb == 0 && tc >= 1 &&
-                !(ok = mbar_wait_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
+                !(ok = mbar_spin_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
               break;
             if (kb == 0) tc_fence_after();
             const uint32_t d_tmem = tmem_base + h * kTmemCols;
@@ -890,11 +942,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       for (int s = 0; s < S && s < iters; ++s) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
-        if (!mbar_wait_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
+        if (!mbar_spin_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
         bool ok = true;
         for (int h = 0; h < 2 && ok; ++h) {
           const int ja = 2 * it + h;
-          ok = mbar_wait(&afull[ja % SA], static_cast<uint32_t>(ja / SA) & 1u, abort_flag, p.err);
+          ok = mbar_spin(&afull[ja % SA], static_cast<uint32_t>(ja / SA) & 1u, abort_flag, p.err);
         }
         if (!ok) break;
         mbar_arrive(&gready[s]);
