@@ -764,7 +764,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint64_t *aempty = afull + SA;      // [SA] pair MMAs reading activation slot a done   (multicast commit)
   uint64_t *empty = aempty + SA;      // [S] pair MMAs reading decoded slot s done       (multicast commit)
   uint64_t *pready = empty + S;       // [S] leader: both weight halves decoded          (1 arrival + st.async tx)
-  uint64_t *gready = pready + S;      // [S] leader: pready and both afull seen by the gate (1 arrival)
+  uint64_t *gready = pready + S;      // [S] leader: pready and half 0's afull seen by the gate (1 arrival)
   uint64_t *cfull = gready + S;       // [SC] this CTA's code tile landed                 (1 arrival + tx)
   uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes      (kDecWarps arrivals)
   uint64_t *tfull = cempty + SC;      // [2] accumulator h of the tile complete          (multicast commit)
@@ -879,10 +879,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
-    // A k-step needs the activation tiles of both halves and both decoded weight
-    // halves, which the gate warp folds into one barrier (gready): every barrier
-    // wait of this thread costs issue time the tensor core cannot hide. For the
-    // same reason no barrier is polled between MMAs.
+    // A k-step needs both decoded weight halves and the activation tile of half 0,
+    // which the gate warp folds into one barrier (gready), and, 8 MMAs later, the
+    // activation tile of half 1 (loaded last, so it gets those 1024 cycles of
+    // slack). Every barrier wait of this thread costs issue time the tensor core
+    // cannot hide, so it spins on the barriers (test_wait) and polls none between MMAs.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
       // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
@@ -893,10 +894,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
                                                 : smem_desc_sw128(smem_u32(ring_b(0)), 16384, 1024);
       int s = 0, a = 0;             // decoded slot of the current k-step, activation slot of its first half
       uint32_t ph = 0;              // phase parity of the decoded slot
-      int tc = 0;
+      int tc = 0, it = 0;           // tiles and k-steps of this cluster so far
       bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
-        for (int kb = 0; kb < num_k; ++kb) {
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
           if (!(ok = mbar_spin(&gready[s], ph, abort_flag, p.err))) break;
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
 #pragma unroll
@@ -906,6 +907,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
                 !(ok = mbar_spin_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
               break;
             if (kb == 0) tc_fence_after();
+            if (h == 1 && !(ok = mbar_spin(&afull[a], static_cast<uint32_t>((2 * it + 1) / SA) & 1u, abort_flag, p.err)))
+              break;
             const uint32_t d_tmem = tmem_base + h * kTmemCols;
             const uint64_t a0 = ad_base + static_cast<uint64_t>(a * (C::kA >> 4));
 #pragma unroll
@@ -933,8 +936,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ gate (leader CTA)
     // Waits, for each k-step, for both decoded halves (pready, a cluster-scope
     // acquire that costs a few hundred cycles even on a completed barrier) and for
-    // the activation tiles of both tile halves (afull), then hands the step to the
-    // MMA thread through one CTA-local barrier. It also arms pready with the signal
+    // the activation tile of half 0 (afull), then hands the step to the MMA thread
+    // through one CTA-local barrier. It also arms pready with the signal
     // bytes of each use (decode warps may signal before it is armed: the missing
     // arrival keeps the phase open).
     if (lane == 0 && rank == 0) {
@@ -943,12 +946,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
         if (!mbar_spin_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
-        bool ok = true;
-        for (int h = 0; h < 2 && ok; ++h) {
-          const int ja = 2 * it + h;
-          ok = mbar_spin(&afull[ja % SA], static_cast<uint32_t>(ja / SA) & 1u, abort_flag, p.err);
-        }
-        if (!ok) break;
+        if (!mbar_spin(&afull[(2 * it) % SA], static_cast<uint32_t>((2 * it) / SA) & 1u, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
