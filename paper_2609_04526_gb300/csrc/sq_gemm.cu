@@ -9,14 +9,16 @@
 // 256-column fp32 accumulators in tensor memory (TMEM), so the epilogue of one
 // tile overlaps the mainloop of the next.
 //
-// FWD / DX (sq_gemm_pair_kernel): a cluster of two CTAs computes a 256 x 256
-// tile with tcgen05.mma.cta_group::2. Each CTA streams its 128 activation rows
-// and its half of the packed-code tile by TMA, and 16 decode warps turn nibbles
-// and scale bytes into the bf16 weight operand directly in the 128B-swizzled
+// FWD / DX (sq_gemm_pair_kernel): a cluster of two CTAs computes a 512 x 256
+// tile with tcgen05.mma.cta_group::2, as two 256-row halves that share every
+// decoded weight stage. Each CTA streams 128 activation rows of each half and
+// its half of the packed-code tile by TMA, and 16 decode warps turn nibbles and
+// scale bytes into the bf16 weight operand directly in the 128B-swizzled
 // shared-memory layout the tensor core reads (K-major for FWD, MN-major for DX).
 //
-// SGRAD (sq_sgrad_kernel): one CTA per 128 x 256 tile of dW = dY^T X with both
-// operands as MN-major TMA tiles; the epilogue reduces code x dW per block.
+// SGRAD (sq_sgrad_pair_kernel): a cluster of two CTAs per 256 x 256 tile of
+// dW = dY^T X with both operands as MN-major TMA tiles; each CTA's epilogue
+// reduces code x dW per block for its 128 rows.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA records
 // kErrWaitTimeout in the device error word, stops issuing, drains what it has
@@ -400,210 +402,13 @@ __device__ __forceinline__ uint32_t load_unit_scale(const KParams &p, int64_t n,
 // E2M1 code and sums every block of B columns, applies the STE mask and writes
 // g[n, b]; the dW tile never leaves the SM.
 
-struct SgradCfg {
-  static constexpr int kEpiWarps = 4;  // warps 0-3: TMEM lanes 0-127
-  static constexpr int kTmaWarp = 4;
-  static constexpr int kMmaWarp = 5;
-  static constexpr int kThreads = 192;
-  static constexpr int kBK = kSgradBK;         // tokens per stage: 4 MMAs of K = 16
-  static constexpr int kStages = 4;
-  static constexpr int kA = kBM * kBK * 2;     // 16 KiB: dY^T tile, two MN atoms of 64 n
-  static constexpr int kB = kBN * kBK * 2;     // 32 KiB: X tile, four MN atoms of 64 k
-  static constexpr int kAtom = kBK * 128;      // bytes of one 64-wide MN atom (kBK rows of 128 B)
-  static constexpr int kStageBytes = kA + kB;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
-};
-
-template <int FMT>
-__global__ void __launch_bounds__(SgradCfg::kThreads, 1)
-    sq_sgrad_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const KParams p) {
-  using C = SgradCfg;
-  constexpr int B = FMT == 0 ? 16 : 32;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kStages * C::kStageBytes);
-  uint64_t *afull = bars;                 // TMA tiles of the stage landed      (1 arrival + tx)
-  uint64_t *empty = bars + C::kStages;       // MMAs reading the stage completed   (tcgen05.commit)
-  uint64_t *tfull = bars + 2 * C::kStages;   // [2] accumulator buffer complete    (tcgen05.commit)
-  uint64_t *tempty = tfull + 2;           // [2] accumulator buffer drained     (kEpiWarps arrivals)
-  uint64_t *drain = tempty + 2;
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int total = p.tiles_m * p.tiles_n;
-  const int num_k = static_cast<int>((p.M + C::kBK - 1) / C::kBK);
-
-  auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
-  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
-
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(&afull[s], 1);
-      mbar_init(&empty[s], 1);
-    }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], C::kEpiWarps);
-    }
-    mbar_init(drain, 1);
-    *abort_flag = 0;
-    fence_barrier_init();
-  }
-  if (warp == C::kMmaWarp) tmem_alloc(tmem_slot, 2 * kTmemCols);
-  if (warp == C::kTmaWarp && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem_base = *tmem_slot;
-
-  if (warp == C::kTmaWarp) {
-    // ------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      int it = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-        int tm, tn;
-        tile_coords<kSgradGroup>(tile, p.tiles_m, p.tiles_n, tm, tn);
-        const int32_t row0 = tm * kBM, col0 = tn * kBN;
-        for (int kb = 0; kb < num_k; ++kb, ++it) {
-          const int s = it % C::kStages;
-          const uint32_t use = static_cast<uint32_t>(it / C::kStages);
-          if (it >= C::kStages && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
-          mbar_arrive_expect_tx(&afull[s], C::kStageBytes);
-          const uint32_t a_dst = smem_u32(stage_a(s));
-          const uint32_t b_dst = smem_u32(stage_b(s));
-          const int32_t kc = kb * C::kBK;
-          for (int j = 0; j < kBM / 64; ++j) tma_load_2d(a_dst + j * C::kAtom, &tmA, &afull[s], row0 + 64 * j, kc);
-          for (int j = 0; j < kBN / 64; ++j) tma_load_2d(b_dst + j * C::kAtom, &tmB, &afull[s], col0 + 64 * j, kc);
-        }
-      }
-      if (*abort_flag) {
-        // Let every issued copy land before the CTA's shared memory goes away.
-        for (int i = (it > C::kStages ? it - C::kStages : 0); i < it; ++i)
-          mbar_drain(&afull[i % C::kStages], static_cast<uint32_t>(i / C::kStages) & 1u);
-      }
-    }
-  } else if (warp == C::kMmaWarp) {
-    // ------------------------------------------------------ MMA issuer
-    // No barrier is polled between the MMAs of a stage: that would hold back their issue.
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(kBM, kBN, 1, 1);
-      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), C::kAtom, 1024);
-      const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), C::kAtom, 1024);
-      int s = 0;
-      uint32_t ph = 0;
-      int tc = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tc) {
-        const int ab = tc & 1;
-        const uint32_t au = static_cast<uint32_t>(tc >> 1);
-        if (tc >= 2 && !(ok = mbar_wait(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + ab * kTmemCols;
-        for (int kb = 0; kb < num_k; ++kb) {
-          if (!(ok = mbar_wait(&afull[s], ph, abort_flag, p.err))) break;
-          const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
-          const uint64_t a0 = ad_base + so, b0 = bd_base + so;
-#pragma unroll
-          for (int kk = 0; kk < C::kBK / 16; ++kk) {
-            umma_bf16(d_tmem, a0 + static_cast<uint64_t>(kk * 2048 >> 4), b0 + static_cast<uint64_t>(kk * 2048 >> 4),
-                      idesc, (kb > 0 || kk > 0) ? 1u : 0u);
-          }
-          umma_commit(&empty[s]);
-          if (++s == C::kStages) {
-            s = 0;
-            ph ^= 1u;
-          }
-        }
-        if (ok) umma_commit(&tfull[ab]);
-      }
-      umma_commit(drain);  // completes once every MMA issued above has finished
-      mbar_drain(drain, 0);
-    }
-  } else {
-    // ------------------------------------------------------ epilogue (warps 0-3)
-    const int r = warp * 32 + lane;
-    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
-    const int64_t G = p.K / B;
-    float *g = static_cast<float *>(p.out);
-    int tc = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++tc) {
-      int tm, tn;
-      tile_coords<kSgradGroup>(tile, p.tiles_m, p.tiles_n, tm, tn);
-      const int64_t n = static_cast<int64_t>(tm) * kBM + r;
-      const int64_t col0 = static_cast<int64_t>(tn) * kBN;
-      const int ab = tc & 1;
-      const uint32_t au = static_cast<uint32_t>(tc >> 1);
-      if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
-      tc_fence_after();
-      const uint32_t t_buf = t_row + ab * kTmemCols;
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(t_buf + c0, v);
-        tmem_ld_wait();
-        const int64_t k = col0 + c0;
-        if (n >= p.N || k >= p.K) continue;
-        const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
-        const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
-        float part[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint32_t o[4];
-          e2m1x8_to_bf16(words[c], o);
-          float acc = 0.f;
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
-            acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
-          }
-          part[c] = acc;
-        }
-        if (FMT == 0) {
-          const int64_t b = k / 16;
-          float g0 = part[0] + part[1];
-          float g1 = part[2] + part[3];
-          if (p.mask) {
-            g0 *= static_cast<float>(p.mask[n * G + b]);
-            g1 *= static_cast<float>(p.mask[n * G + b + 1]);
-          }
-          *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
-        } else {
-          const int64_t b = k / 32;
-          float g0 = (part[0] + part[1]) + (part[2] + part[3]);
-          if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
-          g[n * G + b] = g0;
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[ab]);
-    }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == C::kMmaWarp) {
-    tc_fence_after();
-    tmem_dealloc(tmem_base, 2 * kTmemCols);
-  }
-}
-
-// ------------------------------------------------------------- CTA-pair kernel (FWD / DX)
+// ------------------------------------------------------------- CTA-pair kernels
 //
-// Two CTAs of a cluster share one 256 x 256 output tile through
-// tcgen05.mma.cta_group::2 (M = 256, N = 256): each CTA holds its 128-row half
-// of the activation tile (A) and decodes its 128-row (FWD) or 128-column (DX)
-// half of the weight tile (B), so every SM decodes half as many weights per MMA
-// cycle as in the single-CTA kernel. The leader CTA (cluster rank 0) issues the
-// MMAs; its stage barriers collect the decode warps of both CTAs, and each MMA
-// commit is multicast to the stage / accumulator barriers of both CTAs. Each CTA
-// keeps its 128 accumulator rows in its own TMEM and runs its own epilogue.
+// Two CTAs of a cluster share one output tile through tcgen05.mma.cta_group::2
+// (M = 256, N = 256): each CTA holds 128 rows of the A operand and half (128
+// columns) of the B operand; the leader CTA (cluster rank 0) issues the MMAs and
+// multicasts each commit to the barriers of both CTAs. Each CTA keeps the
+// accumulator of its 128 rows in its own TMEM and runs its own epilogue.
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
@@ -1138,6 +943,229 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   }
 }
 
+// ------------------------------------------------------------- CTA-pair scale-gradient kernel
+//
+// A cluster of two CTAs owns a 256 (n) x 256 (k) tile of dW = dY^T X and issues
+// tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 16 tokens). Each CTA loads 128
+// n-rows of dY^T (A) and 128 k-columns of X (B) per stage, both MN-major, so per
+// MMA each SM reads 8 KiB of operands from its shared memory instead of the
+// 12 KiB of a single-CTA 128 x 256 MMA, and the TMA traffic per SM drops by a
+// third. Each CTA keeps the accumulator of its 128 n-rows (all 256 columns) in
+// its TMEM and reduces it by blocks in its own epilogue.
+struct SgradPairCfg {
+  static constexpr int kEpiWarps = 4;  // warps 0-3: TMEM lanes 0-127
+  static constexpr int kTmaWarp = 4;
+  static constexpr int kMmaWarp = 5;
+  static constexpr int kThreads = 192;
+  static constexpr int kBK = kSgradBK;         // tokens per stage: 4 MMAs of K = 16
+  static constexpr int kStages = 6;
+  static constexpr int kA = 128 * kBK * 2;     // 16 KiB: this CTA's 128 n-rows of dY^T, two MN atoms of 64 n
+  static constexpr int kB = 128 * kBK * 2;     // 16 KiB: this CTA's 128 k-columns of X, two MN atoms of 64 k
+  static constexpr int kAtom = kBK * 128;      // bytes of one 64-wide MN atom (kBK rows of 128 B)
+  static constexpr int kStageBytes = kA + kB;
+  static constexpr uint32_t kTx = 2 * kStageBytes;  // both CTAs' tiles, counted on the leader's barrier
+  static constexpr int kTile = 256;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 1024;
+};
+static_assert(SgradPairCfg::kSmemBytes <= 232448, "scale-gradient kernel exceeds the opt-in shared memory");
+
+template <int FMT>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThreads, 1)
+    sq_sgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                         const KParams p) {
+  using C = SgradPairCfg;
+  constexpr int S = C::kStages;
+  constexpr int B = FMT == 0 ? 16 : 32;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + S * C::kStageBytes);
+  uint64_t *full = bars;              // [S] leader: both CTAs' tiles of the stage landed (1 arrival + tx)
+  uint64_t *empty = full + S;         // [S] pair MMAs reading the stage completed     (multicast commit)
+  uint64_t *tfull = empty + S;        // [2] accumulator buffer complete                (multicast commit)
+  uint64_t *tempty = tfull + 2;       // [2] leader: both epilogues drained the buffer
+                                      //     (kEpiWarps arrivals + the peer warps' st.async tx)
+  uint64_t *drain = tempty + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // [kEpiWarps] leader: st.async targets
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int cluster = blockIdx.x >> 1;
+  const int nclusters = gridDim.x >> 1;
+  const int total = p.tiles_m * p.tiles_n;
+  const int num_k = static_cast<int>((p.M + C::kBK - 1) / C::kBK);
+
+  auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
+  auto stage_b = [&](int s) { return smem + s * C::kStageBytes + C::kA; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], C::kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == C::kMmaWarp) tmem_alloc_pair(tmem_slot, 2 * kTmemCols);
+  if (warp == C::kTmaWarp && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == C::kTmaWarp) {
+    // ------------------------------------------------------ TMA producer (both CTAs)
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        int tm, tn;
+        tile_coords<kSgradGroup>(tile, p.tiles_m, p.tiles_n, tm, tn);
+        const int32_t row0 = tm * C::kTile + 128 * static_cast<int32_t>(rank);  // n
+        const int32_t col0 = tn * C::kTile + 128 * static_cast<int32_t>(rank);  // k
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % S;
+          const uint32_t use = static_cast<uint32_t>(it / S);
+          if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          if (rank == 0) mbar_arrive_expect_tx(&full[s], C::kTx);
+          const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
+          const int32_t kc = kb * C::kBK;
+          for (int j = 0; j < 2; ++j) tma_load_2d_pair(smem_u32(stage_a(s)) + j * C::kAtom, &tmA, bar, row0 + 64 * j, kc);
+          for (int j = 0; j < 2; ++j) tma_load_2d_pair(smem_u32(stage_b(s)) + j * C::kAtom, &tmB, bar, col0 + 64 * j, kc);
+        }
+      }
+      if (*abort_flag && rank == 0) {
+        for (int i = (it > S ? it - S : 0); i < it; ++i) mbar_drain(&full[i % S], static_cast<uint32_t>(i / S) & 1u);
+      }
+    }
+  } else if (warp == C::kMmaWarp) {
+    // ------------------------------------------------------ MMA issuer (leader CTA)
+    // One barrier wait per stage, spinning (test_wait); nothing polled between MMAs.
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 1, 1);
+      const uint64_t ad_base = smem_desc_sw128(smem_u32(stage_a(0)), C::kAtom, 1024);
+      const uint64_t bd_base = smem_desc_sw128(smem_u32(stage_b(0)), C::kAtom, 1024);
+      int s = 0;
+      uint32_t ph = 0;
+      int tc = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
+        const int ab = tc & 1;
+        const uint32_t au = static_cast<uint32_t>(tc >> 1);
+        if (tc >= 2 && !(ok = mbar_spin_cluster(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + ab * kTmemCols;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!(ok = mbar_spin(&full[s], ph, abort_flag, p.err))) break;
+          const uint64_t so = static_cast<uint64_t>(s * (C::kStageBytes >> 4));
+          const uint64_t a0 = ad_base + so, b0 = bd_base + so;
+#pragma unroll
+          for (int kk = 0; kk < C::kBK / 16; ++kk) {
+            // MN-major operands: 16 token rows (2 KiB) per K step
+            umma_bf16_pair(d_tmem, a0 + static_cast<uint64_t>(kk * 2048 >> 4),
+                           b0 + static_cast<uint64_t>(kk * 2048 >> 4), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit_pair_mc(&empty[s]);
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
+        }
+        if (ok) umma_commit_pair_mc(&tfull[ab]);
+      }
+      umma_commit_pair(drain);
+      mbar_drain(drain, 0);
+    }
+  } else if (warp < C::kEpiWarps) {
+    // ------------------------------------------------------ epilogue (warps 0-3, both CTAs)
+    const int r = warp * 32 + lane;
+    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const int64_t G = p.K / B;
+    float *g = static_cast<float *>(p.out);
+    int tc = 0;
+    for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
+      int tm, tn;
+      tile_coords<kSgradGroup>(tile, p.tiles_m, p.tiles_n, tm, tn);
+      const int64_t n = static_cast<int64_t>(tm) * C::kTile + 128 * rank + r;
+      const int64_t col0 = static_cast<int64_t>(tn) * C::kTile;
+      const int ab = tc & 1;
+      const uint32_t au = static_cast<uint32_t>(tc >> 1);
+      if (!mbar_wait(&tfull[ab], au & 1u, abort_flag, p.err)) break;
+      tc_fence_after();
+      const uint32_t t_buf = t_row + ab * kTmemCols;
+      for (int c0 = 0; c0 < C::kTile; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(t_buf + c0, v);
+        tmem_ld_wait();
+        const int64_t k = col0 + c0;
+        if (n >= p.N || k >= p.K) continue;
+        const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(p.codes + n * (p.K / 2) + k / 2));
+        const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+        float part[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[4];
+          e2m1x8_to_bf16(words[c], o);
+          float acc = 0.f;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            acc = fmaf(__uint_as_float(o[e] << 16), __uint_as_float(v[8 * c + 2 * e]), acc);
+            acc = fmaf(__uint_as_float(o[e] & 0xFFFF0000u), __uint_as_float(v[8 * c + 2 * e + 1]), acc);
+          }
+          part[c] = acc;
+        }
+        if (FMT == 0) {
+          const int64_t b = k / 16;
+          float g0 = part[0] + part[1];
+          float g1 = part[2] + part[3];
+          if (p.mask) {
+            g0 *= static_cast<float>(p.mask[n * G + b]);
+            g1 *= static_cast<float>(p.mask[n * G + b + 1]);
+          }
+          *reinterpret_cast<float2 *>(g + n * G + b) = make_float2(g0, g1);
+        } else {
+          const int64_t b = k / 32;
+          float g0 = (part[0] + part[1]) + (part[2] + part[3]);
+          if (p.mask) g0 *= static_cast<float>(p.mask[n * G + b]);
+          g[n * G + b] = g0;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      // buffer drained: the leader's warps arrive (warp 0 arming the peer's bytes),
+      // the peer's warps signal with a non-blocking async store
+      if (lane == 0) {
+        if (rank == 0) {
+          if (warp == 0)
+            mbar_arrive_expect_tx(&tempty[ab], 4 * C::kEpiWarps);
+          else
+            mbar_arrive(&tempty[ab]);
+        } else {
+          st_async_signal(mapa_shared(smem_u32(&sink[warp]), 0), mapa_shared(smem_u32(&tempty[ab]), 0));
+        }
+      }
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync_all();
+  if (warp == C::kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, 2 * kTmemCols);
+  }
+}
+
 template <int MODE, int FMT>
 cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmC, const CUtensorMap *tmOut,
                         int sm_count, cudaStream_t stream) {
@@ -1174,21 +1202,32 @@ cudaError_t launch_pair(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
 template <int FMT>
 cudaError_t launch_sgrad(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, int sm_count,
                          cudaStream_t stream) {
-  using C = SgradCfg;
+  using C = SgradPairCfg;
   static int attr_done_mask = 0;  // per device ordinal (first 31)
+  static int max_clusters[32] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
+  auto kernel = sq_sgrad_pair_kernel<FMT>;
   if (!(attr_done_mask & (1 << (dev & 31)))) {
-    cudaError_t e = cudaFuncSetAttribute(sq_sgrad_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (sm_count / 2), 1, 1);
+    cfg.blockDim = dim3(C::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = sm_count / 2;
+    }
+    max_clusters[dev & 31] = n;
     attr_done_mask |= 1 << (dev & 31);
   }
   KParams p{a.codes, a.scales, a.ws2, a.M, a.N, a.K, a.out, a.mask, a.err,
-            static_cast<int>((a.N + kBM - 1) / kBM), static_cast<int>((a.K + kBN - 1) / kBN)};
+            static_cast<int>((a.N + C::kTile - 1) / C::kTile), static_cast<int>((a.K + C::kTile - 1) / C::kTile)};
   const int64_t total = static_cast<int64_t>(p.tiles_m) * p.tiles_n;
-  const int grid = static_cast<int>(total < sm_count ? total : sm_count);
-  sq_sgrad_kernel<FMT><<<grid, C::kThreads, C::kSmemBytes, stream>>>(tmA, tmB, p);
+  const int64_t nc = total < max_clusters[dev & 31] ? total : max_clusters[dev & 31];
+  kernel<<<static_cast<unsigned>(2 * nc), C::kThreads, C::kSmemBytes, stream>>>(tmA, tmB, p);
   return cudaGetLastError();
 }
 

@@ -14,10 +14,9 @@ enum GemmMode : int {
   MODE_SGRAD = 2   // g  = blockreduce(code * dY^T X)  (GEMM M=out, N=in, contraction=tokens)
 };
 
-// Tile of the scale-gradient kernel: one 128 x 256 fp32 accumulator in TMEM per
-// CTA, kSgradBK tokens per shared-memory stage (also the height of its TMA boxes).
+// Rows of one activation TMA box of the pair kernels (the rows a CTA holds of a tile half).
 constexpr int kBM = 128;
-constexpr int kBN = 256;
+// Tokens per shared-memory stage of the scale-gradient kernel (also the height of its TMA boxes).
 constexpr int kSgradBK = 64;
 
 struct GemmArgs {
