@@ -46,6 +46,10 @@ def parse_args():
     ap.add_argument("--workload", default="c5")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-context", action="store_true",
+                    help="skip the context legs (large-plane projection/merge ceiling, cuBLAS on pre-decoded weights)")
+    ap.add_argument("--plane-only", action="store_true",
+                    help="only the projection/merge ceiling on one 2^28-block plane (for profiling those kernels)")
     return ap.parse_args()
 
 
@@ -309,6 +313,92 @@ def barrier(world):
         torch.distributed.barrier()
 
 
+PLANE_N, PLANE_G = 1 << 18, 1 << 10  # 2^28 scale blocks: far larger than the layer's planes and L2
+
+
+def plane_ceiling(h, pk, stream, reps=10):
+    """Projection and merge over one synthetic 2^28-block NVFP4 plane: at the layer's
+    sizes these launches last a few microseconds, so this shows their HBM ceiling.
+    Bytes per block: projection 4 (latent) + 1 (byte) + 1 (mask); merge 4 + 1 (old
+    byte) + 1 (new byte)."""
+    gen = torch.Generator(device="cuda").manual_seed(2028)
+    ws2 = 1.0 / (6 * 448)
+    L = torch.exp(torch.randn(PLANE_N, PLANE_G, device="cuda", generator=gen) * 2.0 - 3.0) * (448 * ws2 / 20)
+    qb = torch.empty(PLANE_N, PLANE_G, dtype=torch.uint8, device="cuda")
+    mask = torch.empty_like(qb)
+    nonfinite = torch.zeros(1, dtype=torch.int32, device="cuda")
+    art = torch.zeros_like(qb)
+    changed = torch.zeros(1, dtype=torch.int64, device="cuda")
+    blocks = PLANE_N * PLANE_G
+    out = {"blocks": blocks, "shape": [PLANE_N, PLANE_G], "format": "nvfp4"}
+    for name, fn in (("project", lambda: h.sq_project_scales(0, L, ws2, bytes_out=qb, mask_out=mask,
+                                                               nonfinite=nonfinite, stream=stream)),
+                     ("merge", lambda: h.sq_merge(0, L, ws2, art, changed=changed, stream=stream))):
+        for _ in range(3):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        gbs = 6 * blocks / (ms / 1e3) / 1e9
+        out[name] = {"ms": ms, "bytes": 6 * blocks, "achieved": gbs, "unit": "GB/s", "frac": gbs / pk["hbm_gbs"]}
+    h.sq_sync(stream)
+    del L, qb, mask, art
+    return out
+
+
+E2M1_VALUES = (0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0, -0.0, -0.5, -1.0, -1.5, -2.0, -3.0, -4.0, -6.0)
+
+
+def predecoded_weight(wl, st):
+    """The decoded weight as a bf16 tensor (context leg only): codes through the E2M1
+    table times the block scale (E4M3 byte x ws2, or 2^(byte-127))."""
+    codes = st["codes"]
+    nib = torch.stack((codes & 0xF, codes >> 4), dim=-1).reshape(codes.shape[0], -1).long()
+    table = torch.tensor(E2M1_VALUES, dtype=torch.float32, device=codes.device)
+    if wl.fmt == 0:
+        s = st["base_scales"].view(torch.float8_e4m3fn).float() * st["ws2"]
+    else:
+        s = torch.exp2(st["base_scales"].float() - 127.0)
+    return (table[nib] * s.repeat_interleave(wl.block, dim=1)).to(torch.bfloat16)
+
+
+def cublas_context(S, stream, steps=5):
+    """torch.matmul (cuBLAS, bf16 in and out, fp32 accumulation) on pre-decoded weights
+    for the same three contractions per linear: context for the fused kernels, which
+    decode on the fly and reduce dW to g without writing it."""
+    wl = S.wl
+    Ws = [predecoded_weight(wl, st) for st in S.lin]
+    dWs = [torch.empty(st["lin"].N, st["lin"].K, dtype=torch.bfloat16, device="cuda") for st in S.lin]
+    acts = S.acts
+
+    def step():
+        for st, W, dW in zip(S.lin, Ws, dWs):
+            X = acts[st["lin"].x]
+            torch.matmul(X, W.t(), out=st["Y"])
+            torch.matmul(st["dY"], W, out=st["dX"])
+            torch.matmul(st["dY"].t(), X, out=dW)
+
+    for _ in range(2):
+        step()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    del Ws, dWs
+    return {"value": wl.flops() / (ms / 1e3) / 1e12, "unit": UNIT, "ms_per_step": ms,
+            "what": "torch.matmul bf16 on pre-decoded weights (Y, dX and a materialised bf16 dW per linear); "
+                    "context only, not the method"}
+
+
 def run_ours(args):
     import paper_2609_04526_gb300 as pkg
     from paper_2609_04526_gb300 import build, synth
@@ -317,9 +407,13 @@ def run_ours(args):
     build.build()
     wl = synth.WORKLOADS[args.workload]
     pk = peaks()
-    S = LayerState(wl, "cuda")
     h = pkg.Handle()
     stream = torch.cuda.current_stream()
+    if args.plane_only:
+        if rank == 0:
+            print(json.dumps({"plane_ceiling": plane_ceiling(h, pk, stream)}), flush=True)
+        return
+    S = LayerState(wl, "cuda")
     flops_step = wl.flops()
 
     for _ in range(args.warmup):
@@ -417,6 +511,12 @@ def run_ours(args):
                "overlap": "inputs of step k+1 copied on a second stream while step k computes"}
         del sets, host_in
 
+    # ---- context legs: the projection/merge HBM ceiling on a large plane, cuBLAS on pre-decoded weights
+    context = {}
+    if not args.no_context:
+        context["plane_ceiling"] = plane_ceiling(h, pk, stream)
+        context["cublas_context"] = cublas_context(S, stream)
+
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -451,6 +551,7 @@ def run_ours(args):
             "gpu_launches": LAUNCHES_PER_LINEAR * nl * args.steps,
             "clocks": clk,
         }
+        line.update(context)
         print(json.dumps(line), flush=True)
 
 
