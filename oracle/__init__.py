@@ -49,6 +49,12 @@ def lib():
         L.or_dx_at.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _i64, _p, _p, _p]
         L.or_project.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
         L.or_merge.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
+        L.or_lowrank_latent.restype = ctypes.c_float
+        L.or_lowrank_latent.argtypes = [ctypes.c_int, ctypes.c_float, ctypes.c_float, ctypes.c_int, ctypes.c_uint8,
+                                         _p, _p, _i64, _i64]
+        L.or_project_lowrank.argtypes = [ctypes.c_int, _i64, _i64, ctypes.c_int, ctypes.c_float, ctypes.c_float,
+                                         _p, _p, _p, _p, _p, _p, _p]
+        L.or_lowrank_grad.argtypes = [_i64, _i64, ctypes.c_int, ctypes.c_double, _p, _p, _p, _p, _p]
         L.or_num_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -234,3 +240,40 @@ def merge(fmt, latent, scales, ws2, want_delta=True):
     ch = ctypes.c_int64(0)
     lib().or_merge(fmt, L.size, float(ws2), _ptr(L), _ptr(s), _ptr(delta), ctypes.byref(ch))
     return s, delta, int(ch.value)
+
+
+# --- low-rank scale adapter (Sec. 3 "Scale-QLoRA forward") -------------------
+
+def project_lowrank(fmt, base_scales, B_bits, A_bits, ws2, alpha_over_r):
+    """The adapter's latent eff' = eff + (alpha/r) (B A) per block, in fp32 with the
+    order fixed in sq_oracle.c, projected onto the grid (QAST round_grid + clamp).
+    base_scales [N, G] u8; B_bits [N, r] and A_bits [r, G] are bf16 bit patterns.
+    Returns (bytes, mask, nonfinite, latent)."""
+    base = _c(base_scales, np.uint8)
+    B = _c(B_bits, np.uint16)
+    A = _c(A_bits, np.uint16)
+    N, G = base.shape
+    r = B.shape[1]
+    assert B.shape == (N, r) and A.shape == (r, G)
+    out = np.empty((N, G), dtype=np.uint8)
+    mask = np.empty((N, G), dtype=np.uint8)
+    latent = np.empty((N, G), dtype=np.float32)
+    nf = ctypes.c_int(0)
+    lib().or_project_lowrank(fmt, N, G, r, float(ws2), float(alpha_over_r), _ptr(base), _ptr(B), _ptr(A), _ptr(out),
+                             _ptr(mask), ctypes.byref(nf), _ptr(latent))
+    return out, mask, int(nf.value), latent
+
+
+def lowrank_grad(gm, B_bits, A_bits, alpha_over_r):
+    """Adapter gradients from the masked scale gradient gm [N, G] (fp32 values):
+    dB = (alpha/r) gm A^T [N, r] and dA = (alpha/r) B^T gm [r, G], in float64."""
+    g = _c(gm, np.float32)
+    B = _c(B_bits, np.uint16)
+    A = _c(A_bits, np.uint16)
+    N, G = g.shape
+    r = B.shape[1]
+    assert B.shape == (N, r) and A.shape == (r, G)
+    dB = np.empty((N, r), dtype=np.float64)
+    dA = np.empty((r, G), dtype=np.float64)
+    lib().or_lowrank_grad(N, G, r, float(alpha_over_r), _ptr(g), _ptr(B), _ptr(A), _ptr(dB), _ptr(dA))
+    return dB, dA

@@ -353,6 +353,71 @@ void or_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *s
     if (changed) *changed = ch;
 }
 
+/* ------------------------------------------------------------------ */
+/* Low-rank scale adapter (Sec. 3 "Scale-QLoRA forward")                */
+/* ------------------------------------------------------------------ */
+
+/* Latent scale of block (n, b): eff'[n,b] = eff[n,b] + (alpha/r) (B A)[n,b], with
+ * B [N, r] and A [r, G] bf16 (the paper's trainable factors) and the scale
+ * arithmetic in fp32. The paper does not fix the order of the r-term sum; the
+ * reading used on both sides: eff = fl32(decode(base byte) * ws2) (or_scale_f32),
+ * acc = fp32 fused multiply-adds over j = 0 .. r-1 starting from 0, and
+ * eff' = fma(alpha/r, acc, eff) in fp32. Brow = &B[n*r], A is the whole [r, G]. */
+float or_lowrank_latent(int fmt, float ws2, float alpha_over_r, int r, uint8_t base_byte, const uint16_t *Brow,
+                        const uint16_t *A, int64_t G, int64_t b) {
+    float acc = 0.0f;
+    for (int j = 0; j < r; j++) acc = fmaf((float)or_bf16(Brow[j]), (float)or_bf16(A[(int64_t)j * G + b]), acc);
+    return fmaf(alpha_over_r, acc, or_scale_f32(fmt, ws2, base_byte));
+}
+
+/* Projection of the adapter's latent (the grid rounding of the QAST forward,
+ * Sec. 3): for every block, eff' as above, then or_project_one. latent (nullable)
+ * receives eff' in fp32; nonfinite (nullable) the NaN count. */
+void or_project_lowrank(int fmt, int64_t N, int64_t G, int r, float ws2, float alpha_over_r, const uint8_t *base,
+                        const uint16_t *B, const uint16_t *A, uint8_t *bytes, uint8_t *mask, int *nonfinite,
+                        float *latent) {
+    int nan_count = 0;
+    for (int64_t n = 0; n < N; n++) {
+        for (int64_t b = 0; b < G; b++) {
+            const int64_t i = n * G + b;
+            const float L = or_lowrank_latent(fmt, ws2, alpha_over_r, r, base[i], B + n * r, A, G, b);
+            uint8_t by, mk;
+            int isn;
+            or_project_one(fmt, ws2, L, &by, &mk, &isn);
+            bytes[i] = by;
+            if (mask) mask[i] = mk;
+            if (latent) latent[i] = L;
+            nan_count += isn;
+        }
+    }
+    if (nonfinite) *nonfinite = nan_count;
+}
+
+/* Gradients of the adapter factors (Sec. 3: the gradient reaches eff' through the
+ * STE, masked by the ceiling clamp, and eff' is linear in B and in A): with gm the
+ * masked scale gradient [N, G],
+ *   dB[n,j] = (alpha/r) sum_b gm[n,b] A[j,b],   dA[j,b] = (alpha/r) sum_n B[n,j] gm[n,b],
+ * in float64. */
+void or_lowrank_grad(int64_t N, int64_t G, int r, double alpha_over_r, const float *gm, const uint16_t *B,
+                     const uint16_t *A, double *dB, double *dA) {
+#pragma omp parallel for schedule(static)
+    for (int64_t n = 0; n < N; n++) {
+        for (int j = 0; j < r; j++) {
+            double s = 0.0;
+            for (int64_t b = 0; b < G; b++) s += (double)gm[n * G + b] * or_bf16(A[(int64_t)j * G + b]);
+            dB[n * r + j] = alpha_over_r * s;
+        }
+    }
+#pragma omp parallel for schedule(static)
+    for (int64_t b = 0; b < G; b++) {
+        for (int j = 0; j < r; j++) {
+            double s = 0.0;
+            for (int64_t n = 0; n < N; n++) s += or_bf16(B[n * r + j]) * (double)gm[n * G + b];
+            dA[(int64_t)j * G + b] = alpha_over_r * s;
+        }
+    }
+}
+
 int or_num_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();
