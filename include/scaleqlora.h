@@ -9,6 +9,8 @@
  *   sq_scale_grad      g[n,b] = sum_{k in b} code[n,k] (dY^T X)[n,k]   (optionally x mask)
  *   sq_project_scales  latent scale -> on-grid E4M3 / E8M0 byte + STE mask (Sec. 3 QAST, clamp)
  *   sq_merge           write on-grid bytes into the scale plane; never a code (Sec. 3, Sec. 5)
+ *   sq_project_lowrank the low-rank adapter's latent eff + (alpha/r) B A, projected (Sec. 3)
+ *   sq_lowrank_grad    gradients of the adapter factors B and A from the masked scale gradient
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -131,6 +133,40 @@ sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, floa
  * changed_bytes device int64 or NULL: set to the number of bytes that changed. */
 sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
                    uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream);
+
+/* Low-rank scale adapter, Sec. 3 "Scale-QLoRA forward": Delta S = (B A)(alpha/r)
+ * with B [N, r] and A [r, G] (bf16 trainable factors), eff' = eff + Delta S per
+ * block, then the grid projection of sq_project_scales (same clamp, bytes, mask
+ * and NaN count). The latent is formed in fp32 in a fixed order, the same on
+ * every run:
+ *   eff = fl32(E4M3(base byte) * ws2) (NVFP4) or 2^(base byte - 127) (MXFP4);
+ *   acc = fp32 fused multiply-adds over j = 0 .. r-1 from 0 of B[n,j] * A[j,b];
+ *   eff' = fma(alpha_over_r, acc, eff).
+ * base_scales device u8 [N, G] (the frozen base plane, read only); B device bf16
+ * [N, r]; A device bf16 [r, G]; bytes_out device u8 [N, G]; mask_out device u8
+ * [N, G] or NULL; nonfinite device int32 or NULL (set to the NaN count);
+ * latent_out device fp32 [N, G] or NULL (receives eff', e.g. for sq_merge).
+ * Requires 1 <= r <= 256, finite alpha_over_r and the ws2 rule of the format;
+ * N, G in [0, 2^24]; when N or G is 0 only nonfinite is written and the arrays
+ * may be NULL. */
+sq_status sq_project_lowrank(sq_handle h, int32_t fmt, int64_t N, int64_t G, int32_t r, float ws2, float alpha_over_r,
+                             const uint8_t *base_scales, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
+                             uint8_t *mask_out, int32_t *nonfinite, float *latent_out, void *stream);
+
+/* Gradients of the adapter factors (Sec. 3: the gradient reaches eff' through the
+ * straight-through estimator, masked by the ceiling clamp, and eff' is linear in
+ * B and in A). With g the masked scale gradient [N, G] (sq_scale_grad with the
+ * mask of sq_project_lowrank):
+ *   dB[n,j] = alpha_over_r * sum_b g[n,b] A[j,b]    device fp32 [N, r], or NULL
+ *   dA[j,b] = alpha_over_r * sum_n B[n,j] g[n,b]    device fp32 [r, G], or NULL
+ * (not both NULL). fp32 accumulation in a fixed order (the same result on every
+ * run). g device fp32 [N, G]; B device bf16 [N, r]; A device bf16 [r, G].
+ * dA uses scratch in the handle (allocated on first use, grown when needed).
+ * Requires 1 <= r <= 256 and finite alpha_over_r; N, G in [0, 2^24]. An empty
+ * sum gives zeros: with N == 0, dA is zeroed; with G == 0, dB is zeroed; the
+ * arrays of an empty side may be NULL. */
+sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float alpha_over_r, const float *g,
+                          const uint16_t *B, const uint16_t *A, float *dB, float *dA, void *stream);
 
 /* Allocation-free variant of sq_scale_grad. The paper has no counterpart: this
  * entry point exists for callers of this library that cannot call cudaMalloc --

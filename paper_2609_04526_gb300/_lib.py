@@ -26,7 +26,8 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 
 # Every entry point the header declares (checked against include/scaleqlora.h by the tests).
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
-           "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_scale_grad_noalloc")
+           "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
+           "sq_scale_grad_noalloc")
 
 
 class SQError(RuntimeError):
@@ -66,6 +67,8 @@ def load() -> ctypes.CDLL:
     L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
     L.sq_project_scales.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
     L.sq_merge.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
+    L.sq_project_lowrank.argtypes = [vp, i32, i64, i64, i32, f32, f32, vp, vp, vp, vp, vp, vp, vp, vp]
+    L.sq_lowrank_grad.argtypes = [vp, i64, i64, i32, f32, vp, vp, vp, vp, vp, vp]
     L.sq_scale_grad_noalloc.argtypes = [W, vp, vp, i64, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
@@ -174,6 +177,36 @@ class Handle:
         self._check(self._L.sq_project_scales(self._h, fmt, N, G, ws2, _ptr(latent), _ptr(bytes_out), _ptr(mask_out),
                                               _ptr(nonfinite), _stream(stream)))
         return bytes_out, mask_out
+
+    def sq_project_lowrank(self, fmt: int, base_scales: torch.Tensor, B: torch.Tensor, A: torch.Tensor, ws2: float,
+                           alpha_over_r: float, bytes_out: Optional[torch.Tensor] = None,
+                           mask_out: Optional[torch.Tensor] = None, nonfinite: Optional[torch.Tensor] = None,
+                           latent_out: Optional[torch.Tensor] = None, stream=None):
+        """Latent eff + (alpha/r) B A of the low-rank adapter, projected onto the grid.
+        base_scales [N, G] u8; B [N, r] and A [r, G] bf16. Returns (bytes, mask, latent)."""
+        N, G = base_scales.shape
+        r = B.shape[1]
+        if bytes_out is None:
+            bytes_out = torch.empty(N, G, dtype=torch.uint8, device=base_scales.device)
+        self._check(self._L.sq_project_lowrank(self._h, fmt, N, G, r, ws2, alpha_over_r, _ptr(base_scales), _ptr(B),
+                                               _ptr(A), _ptr(bytes_out), _ptr(mask_out), _ptr(nonfinite),
+                                               _ptr(latent_out), _stream(stream)))
+        return bytes_out, mask_out, latent_out
+
+    def sq_lowrank_grad(self, g: torch.Tensor, B: torch.Tensor, A: torch.Tensor, alpha_over_r: float,
+                        dB: Optional[torch.Tensor] = None, dA: Optional[torch.Tensor] = None, want_dB: bool = True,
+                        want_dA: bool = True, stream=None):
+        """dB = (alpha/r) g A^T [N, r] and dA = (alpha/r) B^T g [r, G] (fp32) from the masked
+        scale gradient g [N, G]."""
+        N, G = g.shape
+        r = B.shape[1]
+        if dB is None and want_dB:
+            dB = torch.empty(N, r, dtype=torch.float32, device=g.device)
+        if dA is None and want_dA:
+            dA = torch.empty(r, G, dtype=torch.float32, device=g.device)
+        self._check(self._L.sq_lowrank_grad(self._h, N, G, r, alpha_over_r, _ptr(g), _ptr(B), _ptr(A), _ptr(dB),
+                                            _ptr(dA), _stream(stream)))
+        return dB, dA
 
     def sq_merge(self, fmt: int, latent: torch.Tensor, ws2: float, scales_inout: torch.Tensor,
                  ongrid_delta: Optional[torch.Tensor] = None, changed: Optional[torch.Tensor] = None, stream=None):

@@ -22,7 +22,9 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 struct DeviceState {
   int device;
   int sm_count;
-  int *err_word;  // device int, written by kernels whose bounded waits ran out
+  int *err_word;         // device int, written by kernels whose bounded waits ran out
+  void *workspace;       // scratch of the adapter-gradient kernels, grown on demand
+  size_t workspace_bytes;
 };
 
 constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
@@ -85,7 +87,7 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   int *err_word = nullptr;
   if ((e = cudaMalloc(&err_word, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(error word)");
   if ((e = cudaMemset(err_word, 0, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(error word)");
-  h->devices.push_back(DeviceState{dev, sms, err_word});
+  h->devices.push_back(DeviceState{dev, sms, err_word, nullptr, 0});
   *out = &h->devices.back();
   return SQ_OK;
 }
@@ -227,7 +229,10 @@ sq_status sq_destroy(sq_handle h) {
   int cur = -1;
   cudaGetDevice(&cur);
   for (auto &d : h->devices) {
-    if (cudaSetDevice(d.device) == cudaSuccess) cudaFree(d.err_word);
+    if (cudaSetDevice(d.device) == cudaSuccess) {
+      cudaFree(d.err_word);
+      if (d.workspace) cudaFree(d.workspace);
+    }
   }
   if (cur >= 0) cudaSetDevice(cur);
   delete h;
@@ -315,6 +320,19 @@ sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, cons
   SQ_GUARD_END
 }
 
+// The handle's scratch on the current device, at least `bytes` (a larger buffer
+// replaces the old one; cudaFree waits for the work that may still use it).
+static sq_status ensure_workspace(sq_handle h, DeviceState *dev, size_t bytes) {
+  if (bytes <= dev->workspace_bytes) return SQ_OK;
+  cudaError_t e;
+  if (dev->workspace && (e = cudaFree(dev->workspace)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(workspace)");
+  dev->workspace = nullptr;
+  dev->workspace_bytes = 0;
+  if ((e = cudaMalloc(&dev->workspace, bytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(workspace)");
+  dev->workspace_bytes = bytes;
+  return SQ_OK;
+}
+
 static sq_status check_plane(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2) {
   SQ_TRY(check_ws2(h, fmt, ws2));
   if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
@@ -356,6 +374,72 @@ sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, co
   cudaError_t e = sqi::launch_merge(fmt, N * G, ws2, latent, scales_inout, ongrid_delta, changed_bytes, dev->sm_count,
                                     static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_project_lowrank(sq_handle h, int32_t fmt, int64_t N, int64_t G, int32_t r, float ws2, float alpha_over_r,
+                             const uint8_t *base_scales, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
+                             uint8_t *mask_out, int32_t *nonfinite, float *latent_out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_plane(h, fmt, N, G, ws2));
+  if (r < 1 || r > sqi::kMaxLowRank) return fail(h, SQ_ERR_INVALID_ARG, "rank r=%d must be in [1, 256]", r);
+  if (!std::isfinite(alpha_over_r)) return fail(h, SQ_ERR_INVALID_ARG, "alpha_over_r must be finite");
+  if (nonfinite && (reinterpret_cast<uintptr_t>(nonfinite) & 3u))
+    return fail(h, SQ_ERR_INVALID_ARG, "nonfinite must be 4-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (N == 0 || G == 0) {  // empty plane: the arrays may be NULL
+    if (nonfinite && (e = cudaMemsetAsync(nonfinite, 0, sizeof(int32_t), st)) != cudaSuccess)
+      return cuda_fail(h, e, "cudaMemsetAsync");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, base_scales, "base_scales"));
+  SQ_TRY(check_buf(h, B, "B"));
+  SQ_TRY(check_buf(h, A, "A"));
+  SQ_TRY(check_buf(h, bytes_out, "bytes_out"));
+  if (mask_out && !aligned16(mask_out)) return fail(h, SQ_ERR_INVALID_ARG, "mask_out must be 16-byte aligned");
+  if (latent_out && !aligned16(latent_out)) return fail(h, SQ_ERR_INVALID_ARG, "latent_out must be 16-byte aligned");
+  e = sqi::launch_project_lowrank(fmt, N, G, r, ws2, alpha_over_r, base_scales, B, A, bytes_out, mask_out, nonfinite,
+                                  latent_out, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "adapter projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float alpha_over_r, const float *g,
+                          const uint16_t *B, const uint16_t *A, float *dB, float *dA, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  if (r < 1 || r > sqi::kMaxLowRank) return fail(h, SQ_ERR_INVALID_ARG, "rank r=%d must be in [1, 256]", r);
+  if (!std::isfinite(alpha_over_r)) return fail(h, SQ_ERR_INVALID_ARG, "alpha_over_r must be finite");
+  if (!dB && !dA) return fail(h, SQ_ERR_INVALID_ARG, "dB and dA are both NULL");
+  // dB [N, r] is non-empty iff N > 0 and dA [r, G] iff G > 0; g, B, A are read only when N, G > 0
+  if (dB && N > 0 && !aligned16(dB)) return fail(h, SQ_ERR_INVALID_ARG, "dB must be non-NULL and 16-byte aligned");
+  if (dA && G > 0 && !aligned16(dA)) return fail(h, SQ_ERR_INVALID_ARG, "dA must be non-NULL and 16-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (N == 0 || G == 0) {  // empty sums: the gradients are zero
+    if (dB && N > 0 && (e = cudaMemsetAsync(dB, 0, static_cast<size_t>(N) * r * sizeof(float), st)) != cudaSuccess)
+      return cuda_fail(h, e, "cudaMemsetAsync");
+    if (dA && G > 0 && (e = cudaMemsetAsync(dA, 0, static_cast<size_t>(G) * r * sizeof(float), st)) != cudaSuccess)
+      return cuda_fail(h, e, "cudaMemsetAsync");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, g, "g"));
+  SQ_TRY(check_buf(h, B, "B"));
+  SQ_TRY(check_buf(h, A, "A"));
+  if (dA) SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r)));
+  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
+                               dev->sm_count, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");
   return SQ_OK;
   SQ_GUARD_END
 }

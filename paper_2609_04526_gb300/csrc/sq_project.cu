@@ -210,6 +210,169 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   if (changed) warp_add_i64(changed, n_changed);
 }
 
+// ---------------------------------------------------------------- low-rank scale adapter
+//
+// Sec. 3 "Scale-QLoRA forward": the latent block scale eff' = eff + (alpha/r) (B A),
+// B [N, r] and A [r, G] bf16, formed in fp32 in a fixed order -- eff = fl32(decoded
+// base byte * ws2) (scale_value), acc = fused multiply-adds over j = 0 .. r-1 from 0,
+// eff' = fma(alpha/r, acc, eff) -- and projected exactly as sq_project_kernel. A CTA
+// owns a 32 x 64 block of the plane with its 32 B rows and 64 A columns staged in
+// shared memory; each thread accumulates 4 rows x 2 columns (the B values are warp
+// broadcasts, the A values consecutive).
+constexpr int kLrRows = 32;
+constexpr int kLrCols = 64;
+
+__device__ __forceinline__ float bf16_bits(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
+    int64_t N, int64_t G, int r, float ws2, float cap, float aor, const uint8_t *__restrict__ base,
+    const uint16_t *__restrict__ B, const uint16_t *__restrict__ A, uint8_t *__restrict__ bytes_out,
+    uint8_t *__restrict__ mask_out, int32_t *__restrict__ nonfinite, float *__restrict__ latent_out) {
+  extern __shared__ uint16_t lr_smem[];
+  uint16_t *sB = lr_smem;                // [kLrRows][r]
+  uint16_t *sA = lr_smem + kLrRows * r;  // [r][kLrCols]
+  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kLrRows;
+  const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kLrCols;
+  for (int i = threadIdx.x; i < kLrRows * r; i += kThreads) {
+    const int64_t n = n0 + i / r;
+    sB[i] = n < N ? B[n * r + i % r] : static_cast<uint16_t>(0);
+  }
+  for (int i = threadIdx.x; i < r * kLrCols; i += kThreads) {
+    const int64_t b = b0 + i % kLrCols;
+    sA[i] = b < G ? A[static_cast<int64_t>(i / kLrCols) * G + b] : static_cast<uint16_t>(0);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float acc[4][2];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) acc[q][0] = acc[q][1] = 0.f;
+  for (int j = 0; j < r; ++j) {
+    const float a0 = bf16_bits(sA[j * kLrCols + lane]);
+    const float a1 = bf16_bits(sA[j * kLrCols + 32 + lane]);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float bq = bf16_bits(sB[(warp * 4 + q) * r + j]);
+      acc[q][0] = fmaf(bq, a0, acc[q][0]);
+      acc[q][1] = fmaf(bq, a1, acc[q][1]);
+    }
+  }
+  uint32_t nan_count = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const int64_t n = n0 + warp * 4 + q, b = b0 + lane + 32 * c;
+      if (n < N && b < G) {
+        const int64_t i = n * G + b;
+        const float L = fmaf(aor, acc[q][c], scale_value<FMT>(base[i], ws2));
+        uint32_t by, mk, na;
+        project_one<FMT>(L, ws2, cap, by, mk, na);
+        bytes_out[i] = static_cast<uint8_t>(by);
+        if (mask_out) mask_out[i] = static_cast<uint8_t>(mk);
+        if (latent_out) latent_out[i] = L;
+        nan_count += na;
+      }
+    }
+  }
+  if (nonfinite) warp_add_i32(nonfinite, nan_count);
+}
+
+// Adapter gradients from the masked scale gradient g [N, G]: dB[n,j] = (alpha/r) sum_b
+// g[n,b] A[j,b] and dA[j,b] = (alpha/r) sum_n B[n,j] g[n,b], fp32 accumulation in a fixed
+// order (the same result on every run).
+//
+// dB: one warp per row n, 32 j at a time; each lane sums over the columns b = lane
+// (mod 32) of 256-column chunks of A staged in shared memory, then a butterfly sums
+// the lanes.
+constexpr int kDbChunk = 256;
+constexpr int kWarps = kThreads / 32;
+
+__global__ void __launch_bounds__(kThreads) sq_lowrank_db_kernel(int64_t N, int64_t G, int r, float aor,
+                                                                 const float *__restrict__ g,
+                                                                 const uint16_t *__restrict__ A,
+                                                                 float *__restrict__ dB) {
+  extern __shared__ uint16_t db_smem[];  // [r][kDbChunk] chunk of A
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t n = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+  for (int jc = 0; jc < r; jc += 32) {
+    const int nj = min(32, r - jc);
+    float acc[32];
+#pragma unroll
+    for (int t = 0; t < 32; ++t) acc[t] = 0.f;
+    for (int64_t bc = 0; bc < G; bc += kDbChunk) {
+      const int w = G - bc < kDbChunk ? static_cast<int>(G - bc) : kDbChunk;
+      __syncthreads();
+      for (int i = threadIdx.x; i < nj * kDbChunk; i += kThreads) {
+        const int t = i / kDbChunk, c = i % kDbChunk;
+        db_smem[i] = c < w ? A[static_cast<int64_t>(jc + t) * G + bc + c] : static_cast<uint16_t>(0);
+      }
+      __syncthreads();
+      if (n < N) {
+        for (int c = lane; c < w; c += 32) {
+          const float gv = g[n * G + bc + c];
+#pragma unroll
+          for (int t = 0; t < 32; ++t)
+            if (t < nj) acc[t] = fmaf(gv, bf16_bits(db_smem[t * kDbChunk + c]), acc[t]);
+        }
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < 32; ++t) {
+      float v = acc[t];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+      if (n < N && lane == t && t < nj) dB[n * r + jc + t] = aor * v;
+    }
+  }
+}
+
+// dA, pass 1: a CTA takes kDaRows rows n and 32 columns b; lane = column, warp w takes
+// j = w, w + 8, ...; the rows are summed in order into partial[chunk][j][b].
+constexpr int kDaRows = 128;
+constexpr int kDaJ = 32;  // accumulators per thread: r <= 8 * kDaJ = 256
+
+__global__ void __launch_bounds__(kThreads) sq_lowrank_da_partial_kernel(int64_t N, int64_t G, int r,
+                                                                         const float *__restrict__ g,
+                                                                         const uint16_t *__restrict__ B,
+                                                                         float *__restrict__ partial) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t chunk = blockIdx.x;
+  const int64_t b = static_cast<int64_t>(blockIdx.y) * 32 + lane;
+  const int64_t n0 = chunk * kDaRows, n1 = N < n0 + kDaRows ? N : n0 + kDaRows;
+  float acc[kDaJ];
+#pragma unroll
+  for (int t = 0; t < kDaJ; ++t) acc[t] = 0.f;
+  for (int64_t n = n0; n < n1; ++n) {
+    const float gv = b < G ? g[n * G + b] : 0.f;
+#pragma unroll
+    for (int t = 0; t < kDaJ; ++t) {
+      const int j = warp + kWarps * t;
+      if (j < r) acc[t] = fmaf(bf16_bits(B[n * r + j]), gv, acc[t]);
+    }
+  }
+  if (b < G) {
+#pragma unroll
+    for (int t = 0; t < kDaJ; ++t) {
+      const int j = warp + kWarps * t;
+      if (j < r) partial[(chunk * r + j) * G + b] = acc[t];
+    }
+  }
+}
+
+// dA, pass 2: dA[j,b] = (alpha/r) * sum over chunks, in chunk order.
+__global__ void __launch_bounds__(kThreads) sq_lowrank_da_reduce_kernel(int64_t G, int r, int64_t chunks, float aor,
+                                                                        const float *__restrict__ partial,
+                                                                        float *__restrict__ dA) {
+  const int64_t count = static_cast<int64_t>(r) * G;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < count;
+       i += static_cast<int64_t>(gridDim.x) * kThreads) {
+    float s = 0.f;
+    for (int64_t c = 0; c < chunks; ++c) s += partial[c * count + i];
+    dA[i] = aor * s;
+  }
+}
+
 unsigned grid_for(int64_t count, int sm_count) {
   const int64_t nvec = count / 16;
   const int64_t want = (nvec + kThreads - 1) / kThreads;
@@ -251,6 +414,56 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
   else
     sq_merge_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, latent, scales_inout, ongrid_delta, changed);
   return cudaGetLastError();
+}
+
+cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float ws2, float alpha_over_r,
+                                   const uint8_t *base, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
+                                   uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream) {
+  if (nonfinite) {
+    cudaError_t e = cudaMemsetAsync(nonfinite, 0, sizeof(int32_t), stream);
+    if (e != cudaSuccess) return e;
+  }
+  const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
+  const dim3 grid(static_cast<unsigned>((N + kLrRows - 1) / kLrRows), static_cast<unsigned>((G + kLrCols - 1) / kLrCols));
+  const size_t smem = static_cast<size_t>(kLrRows + kLrCols) * r * sizeof(uint16_t);
+  if (fmt == 0)
+    sq_project_lowrank_kernel<0><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
+                                                                   bytes_out, mask_out, nonfinite, latent_out);
+  else
+    sq_project_lowrank_kernel<1><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
+                                                                   bytes_out, mask_out, nonfinite, latent_out);
+  return cudaGetLastError();
+}
+
+size_t lowrank_grad_workspace(int64_t N, int64_t G, int r) {
+  const int64_t chunks = (N + kDaRows - 1) / kDaRows;
+  return static_cast<size_t>(chunks) * r * G * sizeof(float);
+}
+
+cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
+                                const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
+                                cudaStream_t stream) {
+  if (dB) {
+    const unsigned grid = static_cast<unsigned>((N + kWarps - 1) / kWarps);
+    const size_t smem = static_cast<size_t>(min(r, 32)) * kDbChunk * sizeof(uint16_t);
+    sq_lowrank_db_kernel<<<grid, kThreads, smem, stream>>>(N, G, r, alpha_over_r, g, A, dB);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  if (dA) {
+    const int64_t chunks = (N + kDaRows - 1) / kDaRows;
+    const dim3 grid1(static_cast<unsigned>(chunks), static_cast<unsigned>((G + 31) / 32));
+    sq_lowrank_da_partial_kernel<<<grid1, kThreads, 0, stream>>>(N, G, r, g, B, workspace);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t count = static_cast<int64_t>(r) * G;
+    int64_t blocks = (count + kThreads - 1) / kThreads;
+    if (blocks > static_cast<int64_t>(sm_count) * kCtasPerSm) blocks = static_cast<int64_t>(sm_count) * kCtasPerSm;
+    sq_lowrank_da_reduce_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(G, r, chunks, alpha_over_r,
+                                                                                      workspace, dA);
+    return cudaGetLastError();
+  }
+  return cudaSuccess;
 }
 
 }  // namespace sqi

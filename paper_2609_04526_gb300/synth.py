@@ -18,6 +18,8 @@ import dataclasses
 import zlib
 from typing import Dict, List, Optional
 
+import math
+
 import torch
 
 NVFP4 = 0
@@ -216,6 +218,26 @@ def gen_latent(wl: Workload, lin: Linear, weight: Weight, device="cpu") -> torch
         hot = torch.rand(N, G, generator=g, device=device) < wl.above_ceiling_frac
         L = torch.where(hot, cap * (1.0 + 0.5 * u), L)
     return L.contiguous()
+
+
+def gen_adapter(wl: Workload, lin: Linear, weight: Weight, r: int = 58, alpha: float = 16.0, device="cpu"):
+    """Low-rank scale adapter factors in mid-training: B [N, r] and A [r, G] bf16 and
+    alpha/r (the adapter of Sec. 3 "Scale-QLoRA forward"; r = 58 is the paper's
+    Llama-8B rank). Seeded Gaussians, A ~ N(0, 1/r) and B scaled so (alpha/r) (B A)
+    has the workload's latent relative RMS of the median effective scale, so a few
+    percent of bytes move. Returns (B, A, alpha_over_r)."""
+    N, G = weight.scales.shape
+    g = _gen(wl.seed, "adapter:" + lin.name, device)
+    sb = weight.scales.to(device)
+    if wl.fmt == NVFP4:
+        s = sb.view(torch.float8_e4m3fn).to(torch.float32) * weight.ws2
+    else:
+        s = torch.ldexp(torch.ones(N, G, device=device), sb.to(torch.int32) - 127)
+    aor = alpha / r
+    s_med = float(s.abs().float().median().clamp(min=1e-30))
+    A = torch.randn(r, G, generator=g, device=device) / math.sqrt(r)
+    B = torch.randn(N, r, generator=g, device=device) * (wl.latent_rel_rms * s_med / aor)
+    return B.to(torch.bfloat16).contiguous(), A.to(torch.bfloat16).contiguous(), aor
 
 
 def act_names(wl: Workload) -> List[str]:
