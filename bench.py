@@ -35,6 +35,8 @@ import torch  # noqa: E402
 METRIC = "fwd+dX+dScale TFLOP/s per layer & fraction of GB300 bf16 tensor peak"
 UNIT = "TFLOP/s"
 KINDS = ("project", "fwd", "dx", "sgrad", "merge")
+KINDS_LOWRANK = ("project", "fwd", "dx", "sgrad", "adapter_grad", "merge")
+ADAPTER_RANK = 58  # the paper's Llama-3-8B scale rank (Sec. 5 recipe)
 
 
 def parse_args():
@@ -50,6 +52,10 @@ def parse_args():
                     help="skip the context legs (large-plane projection/merge ceiling, cuBLAS on pre-decoded weights)")
     ap.add_argument("--plane-only", action="store_true",
                     help="only the projection/merge ceiling on one 2^28-block plane (for profiling those kernels)")
+    ap.add_argument("--lowrank", action="store_true",
+                    help="the paper's exact training step: the latent comes from the low-rank adapter "
+                         "(sq_project_lowrank) and the adapter gradients follow the scale gradient "
+                         "(device-resident step only: no e2e or CPU-baseline legs)")
     return ap.parse_args()
 
 
@@ -140,10 +146,11 @@ class ClockSampler:
 class LayerState:
     """Device-resident inputs and outputs of one step of the workload."""
 
-    def __init__(self, wl, device):
+    def __init__(self, wl, device, lowrank=False):
         import paper_2609_04526_gb300 as pkg
         from paper_2609_04526_gb300 import synth
         self.wl = wl
+        self.lowrank = lowrank
         self.lin = []
         self.acts = {name: synth.gen_act(wl, name, device=device) for name in synth.act_names(wl)}
         for lin in wl.linears:
@@ -163,6 +170,10 @@ class LayerState:
                 changed=torch.zeros(1, dtype=torch.int64, device=device),
             )
             st["qw"] = pkg.QuantWeight(wl.fmt, lin.N, lin.K, w.codes, st["qbytes"], w.ws2)
+            if lowrank:
+                st["B"], st["A"], st["aor"] = synth.gen_adapter(wl, lin, w, r=ADAPTER_RANK, device=device)
+                st["dB"] = torch.empty(lin.N, ADAPTER_RANK, dtype=torch.float32, device=device)
+                st["dA"] = torch.empty(ADAPTER_RANK, G, dtype=torch.float32, device=device)
             self.lin.append(st)
 
     def results(self):
@@ -191,7 +202,9 @@ def flat_inputs(ins):
 
 def run_step(h, S, stream, events=None, ins=None):
     """One step over every linear: projection (+ STE mask), forward, input gradient,
-    masked scale gradient, merge into the artifact scale plane."""
+    masked scale gradient, merge into the artifact scale plane. With the low-rank
+    adapter (S.lowrank) the latent is formed from the adapter inside the projection
+    (and kept for the merge), and the adapter gradients follow the scale gradient."""
     fmt = S.wl.fmt
     ins = input_set(S) if ins is None else ins
     for i, st in enumerate(S.lin):
@@ -199,27 +212,38 @@ def run_step(h, S, stream, events=None, ins=None):
         dY = ins["dY"][i]
         L = ins["L"][i]
         ev = events[i] if events is not None else None
-        if ev:
-            ev[0].record(stream)
-        h.sq_project_scales(fmt, L, st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
-                            nonfinite=st["nonfinite"], stream=stream)
-        if ev:
-            ev[1].record(stream)
+        e = 0
+
+        def mark():
+            nonlocal e
+            if ev:
+                ev[e].record(stream)
+            e += 1
+
+        mark()
+        if S.lowrank:
+            h.sq_project_lowrank(fmt, st["base_scales"], st["B"], st["A"], st["ws2"], st["aor"],
+                                 bytes_out=st["qbytes"], mask_out=st["mask"], nonfinite=st["nonfinite"],
+                                 latent_out=L, stream=stream)
+        else:
+            h.sq_project_scales(fmt, L, st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
+                                nonfinite=st["nonfinite"], stream=stream)
+        mark()
         h.sq_fwd(st["qw"], X, st["Y"], stream=stream)
-        if ev:
-            ev[2].record(stream)
+        mark()
         h.sq_bwd_dx(st["qw"], dY, st["dX"], stream=stream)
-        if ev:
-            ev[3].record(stream)
+        mark()
         h.sq_scale_grad(st["qw"], X, dY, mask=st["mask"], g=st["g"], stream=stream)
-        if ev:
-            ev[4].record(stream)
+        mark()
+        if S.lowrank:
+            h.sq_lowrank_grad(st["g"], st["B"], st["A"], st["aor"], dB=st["dB"], dA=st["dA"], stream=stream)
+            mark()
         h.sq_merge(fmt, L, st["ws2"], st["art"], changed=st["changed"], stream=stream)
-        if ev:
-            ev[5].record(stream)
+        mark()
 
 
 LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge kernels
+LAUNCHES_PER_LINEAR_LOWRANK = 8  # + the adapter gradients' three kernels (dB, dA partials, dA reduce)
 
 
 def kernel_work(S):
@@ -231,8 +255,14 @@ def kernel_work(S):
         for k in fl:
             fl[k] += 2 * S.wl.M * l.N * l.K
         blocks = l.N * (l.K // S.wl.block)
-        by["project"] += blocks * (4 + 1 + 1)   # latent fp32 in, byte + mask byte out
         by["merge"] += blocks * (4 + 1 + 1)     # latent in, old byte in, new byte out
+        if S.lowrank:
+            r = ADAPTER_RANK
+            factors = (l.N * r + r * (l.K // S.wl.block)) * 2   # B and A, bf16
+            by["project"] += blocks * (1 + 1 + 1 + 4) + factors  # base byte in; byte, mask, latent out
+            by["adapter_grad"] = by.get("adapter_grad", 0) + blocks * 4 + factors + factors * 2  # g in; dB, dA fp32 out
+        else:
+            by["project"] += blocks * (4 + 1 + 1)   # latent fp32 in, byte + mask byte out
     return fl, by
 
 
@@ -367,6 +397,56 @@ def predecoded_weight(wl, st):
     return (table[nib] * s.repeat_interleave(wl.block, dim=1)).to(torch.bfloat16)
 
 
+def adapter_leg(h, S, stream, reps=10):
+    """The low-rank adapter kernels alone over the layer's linears (rank 58): the
+    adapter projection (latent formed from B, A and projected, with mask and latent
+    out) and the adapter gradients (dB, dA from the masked scale gradient). GB/s
+    from their algorithmic bytes."""
+    from paper_2609_04526_gb300 import synth
+    wl = S.wl
+    r = ADAPTER_RANK
+    per = []
+    by_proj = by_grad = 0
+    for st in S.lin:
+        l = st["lin"]
+        G = l.K // wl.block
+        w = synth.Weight(wl.fmt, l.N, l.K, st["codes"], st["base_scales"], st["ws2"])
+        B, A, aor = synth.gen_adapter(wl, l, w, r=r, device="cuda")
+        per.append(dict(st=st, B=B, A=A, aor=aor, L=torch.empty(l.N, G, dtype=torch.float32, device="cuda"),
+                        q=torch.empty(l.N, G, dtype=torch.uint8, device="cuda"),
+                        m=torch.empty(l.N, G, dtype=torch.uint8, device="cuda"),
+                        dB=torch.empty(l.N, r, dtype=torch.float32, device="cuda"),
+                        dA=torch.empty(r, G, dtype=torch.float32, device="cuda")))
+        blocks, factors = l.N * G, (l.N * r + r * G) * 2
+        by_proj += blocks * (1 + 1 + 1 + 4) + factors
+        by_grad += blocks * 4 + factors + factors * 2
+
+    def proj():
+        for a in per:
+            h.sq_project_lowrank(wl.fmt, a["st"]["base_scales"], a["B"], a["A"], a["st"]["ws2"], a["aor"],
+                                 bytes_out=a["q"], mask_out=a["m"], latent_out=a["L"], stream=stream)
+
+    def grad():
+        for a in per:
+            h.sq_lowrank_grad(a["st"]["g"], a["B"], a["A"], a["aor"], dB=a["dB"], dA=a["dA"], stream=stream)
+
+    out = {"rank": r, "linears": len(per)}
+    for name, fn, by in (("project_lowrank", proj, by_proj), ("adapter_grad", grad, by_grad)):
+        for _ in range(3):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        out[name] = {"us_per_layer": ms * 1e3, "bytes": by, "achieved": by / (ms / 1e3) / 1e9, "unit": "GB/s"}
+    h.sq_sync(stream)
+    return out
+
+
 def cublas_context(S, stream, steps=5):
     """torch.matmul (cuBLAS, bf16 in and out, fp32 accumulation) on pre-decoded weights
     for the same three contractions per linear: context for the fused kernels, which
@@ -413,7 +493,11 @@ def run_ours(args):
         if rank == 0:
             print(json.dumps({"plane_ceiling": plane_ceiling(h, pk, stream)}), flush=True)
         return
-    S = LayerState(wl, "cuda")
+    if args.lowrank:
+        args.no_e2e = True
+        args.no_cpu_baseline = True
+    kinds = KINDS_LOWRANK if args.lowrank else KINDS
+    S = LayerState(wl, "cuda", lowrank=args.lowrank)
     flops_step = wl.flops()
 
     for _ in range(args.warmup):
@@ -422,7 +506,8 @@ def run_ours(args):
 
     # ---- device-resident timed region (inputs already in HBM; inputs > L2)
     nl = len(S.lin)
-    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(nl)] for _ in range(args.steps)]
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(len(kinds) + 1)] for _ in range(nl)]
+              for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize()
@@ -438,17 +523,17 @@ def run_ours(args):
     ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
     ms_step = ms_total / args.steps
 
-    kind_ms = {k: 0.0 for k in KINDS}
-    kind_launch = {k: 0 for k in KINDS}
+    kind_ms = {k: 0.0 for k in kinds}
+    kind_launch = {k: 0 for k in kinds}
     for k in range(args.steps):
         for i in range(nl):
             ev = events[k][i]
-            for j, kind in enumerate(KINDS):
+            for j, kind in enumerate(kinds):
                 kind_ms[kind] += ev[j].elapsed_time(ev[j + 1])
                 kind_launch[kind] += 1
     fl, by = kernel_work(S)
     kernels = {}
-    for kind in KINDS:
+    for kind in kinds:
         t = kind_ms[kind] / args.steps / 1e3  # s per step
         if kind in fl:
             ach = fl[kind] / t / 1e12
@@ -458,8 +543,8 @@ def run_ours(args):
             ach = by[kind] / t / 1e9
             kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
     dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
-    traffic = profiled_traffic(wl.key)
-    for kind in KINDS:
+    traffic = {} if args.lowrank else profiled_traffic(wl.key)  # the profile is of the default step's kernels
+    for kind in kinds:
         if kind in traffic:
             kernels[kind]["dram_bytes_per_launch"] = traffic[kind]["dram_bytes_per_launch"]
     value = flops_step * args.steps * world / (ms_total / 1e3) / 1e12
@@ -515,6 +600,7 @@ def run_ours(args):
     context = {}
     if not args.no_context:
         context["plane_ceiling"] = plane_ceiling(h, pk, stream)
+        context["adapter_kernels"] = adapter_leg(h, S, stream)
         context["cublas_context"] = cublas_context(S, stream)
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
@@ -537,7 +623,9 @@ def run_ours(args):
             "config": {"workload": f"{wl.key}: {wl.title}", "M": wl.M,
                        "linears": {l.name: [l.N, l.K] for l in wl.linears}, "format": "nvfp4" if wl.fmt == 0 else "mxfp4",
                        "l2": "inputs larger than L2 (activations + output gradients > 4 GB per step), no flush",
-                       "parallelism": f"replicas x{world}", "flops_per_step": flops_step},
+                       "parallelism": f"replicas x{world}", "flops_per_step": flops_step,
+                       "step": (f"adapter step: latent from a rank-{ADAPTER_RANK} scale adapter, adapter gradients"
+                                if args.lowrank else "latent projection")},
             "roofline": {"bound": "tensor", "kernel": dom, "achieved": k["achieved"],
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": k["achieved"] / pk["bf16_sustained"],
                          "traffic": traffic.get(dom, {}).get("dram_bytes_per_launch"),
@@ -548,7 +636,7 @@ def run_ours(args):
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels,
             "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": LAUNCHES_PER_LINEAR * nl * args.steps,
+            "gpu_launches": (LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl * args.steps,
             "clocks": clk,
         }
         line.update(context)

@@ -436,7 +436,7 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
   SQ_TRY(check_buf(h, g, "g"));
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
-  if (dA) SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r)));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count)));
   e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
                                dev->sm_count, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");

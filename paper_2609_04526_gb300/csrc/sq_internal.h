@@ -46,11 +46,11 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
 
 // Low-rank scale adapter (Sec. 3 "Scale-QLoRA forward"): latent eff + (alpha/r) B A
 // projected onto the grid; and the gradients of B and A from the masked scale
-// gradient. The gradient of A uses `workspace` (lowrank_grad_workspace bytes).
+// gradient, through `workspace` (lowrank_grad_workspace bytes).
 cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float ws2, float alpha_over_r,
                                    const uint8_t *base, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
                                    uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream);
-size_t lowrank_grad_workspace(int64_t N, int64_t G, int r);
+size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count);
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
                                 cudaStream_t stream);

@@ -7,6 +7,8 @@
 // store, and the grid is a whole number of waves over the SMs (grid-stride).
 // Counters (NaN latents, changed bytes) are reduced within each warp and added
 // with one atomic per warp.
+#include <algorithm>
+
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
 
@@ -215,12 +217,13 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
 // Sec. 3 "Scale-QLoRA forward": the latent block scale eff' = eff + (alpha/r) (B A),
 // B [N, r] and A [r, G] bf16, formed in fp32 in a fixed order -- eff = fl32(decoded
 // base byte * ws2) (scale_value), acc = fused multiply-adds over j = 0 .. r-1 from 0,
-// eff' = fma(alpha/r, acc, eff) -- and projected exactly as sq_project_kernel. A CTA
-// owns a 32 x 64 block of the plane with its 32 B rows and 64 A columns staged in
-// shared memory; each thread accumulates 4 rows x 2 columns (the B values are warp
-// broadcasts, the A values consecutive).
-constexpr int kLrRows = 32;
-constexpr int kLrCols = 64;
+// eff' = fma(alpha/r, acc, eff) -- and projected exactly as sq_project_kernel.
+// The three adapter kernels are register-tiled fp32 CUDA-core products: a CTA of 256
+// threads owns a 64 x 64 output tile, its operands staged in shared memory as fp32,
+// and each thread accumulates a 4 x 4 sub-tile (rows ty*4 .. +3, columns tx + 16c),
+// so 8 shared-memory loads feed 16 fused multiply-adds. Every output is summed
+// sequentially over the contraction index, so results do not change between runs.
+constexpr int kT = 64;  // output tile edge
 
 __device__ __forceinline__ float bf16_bits(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
 
@@ -229,40 +232,43 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
     int64_t N, int64_t G, int r, float ws2, float cap, float aor, const uint8_t *__restrict__ base,
     const uint16_t *__restrict__ B, const uint16_t *__restrict__ A, uint8_t *__restrict__ bytes_out,
     uint8_t *__restrict__ mask_out, int32_t *__restrict__ nonfinite, float *__restrict__ latent_out) {
-  extern __shared__ uint16_t lr_smem[];
-  uint16_t *sB = lr_smem;                // [kLrRows][r]
-  uint16_t *sA = lr_smem + kLrRows * r;  // [r][kLrCols]
-  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kLrRows;
-  const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kLrCols;
-  for (int i = threadIdx.x; i < kLrRows * r; i += kThreads) {
+  extern __shared__ float lr_smem[];
+  float *sB = lr_smem;            // [kT rows][r]
+  float *sA = lr_smem + kT * r;   // [r][kT columns]
+  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kT;
+  const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kT;
+  for (int i = threadIdx.x; i < kT * r; i += kThreads) {
     const int64_t n = n0 + i / r;
-    sB[i] = n < N ? B[n * r + i % r] : static_cast<uint16_t>(0);
+    sB[i] = n < N ? bf16_bits(B[n * r + i % r]) : 0.f;
   }
-  for (int i = threadIdx.x; i < r * kLrCols; i += kThreads) {
-    const int64_t b = b0 + i % kLrCols;
-    sA[i] = b < G ? A[static_cast<int64_t>(i / kLrCols) * G + b] : static_cast<uint16_t>(0);
+  for (int i = threadIdx.x; i < r * kT; i += kThreads) {
+    const int64_t b = b0 + i % kT;
+    sA[i] = b < G ? bf16_bits(A[static_cast<int64_t>(i / kT) * G + b]) : 0.f;
   }
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float acc[4][2];
+  const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+  float acc[4][4];
 #pragma unroll
-  for (int q = 0; q < 4; ++q) acc[q][0] = acc[q][1] = 0.f;
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[q][c] = 0.f;
   for (int j = 0; j < r; ++j) {
-    const float a0 = bf16_bits(sA[j * kLrCols + lane]);
-    const float a1 = bf16_bits(sA[j * kLrCols + 32 + lane]);
+    float bv[4], av[4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float bq = bf16_bits(sB[(warp * 4 + q) * r + j]);
-      acc[q][0] = fmaf(bq, a0, acc[q][0]);
-      acc[q][1] = fmaf(bq, a1, acc[q][1]);
-    }
+    for (int q = 0; q < 4; ++q) bv[q] = sB[(ty * 4 + q) * r + j];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) av[c] = sA[j * kT + tx + 16 * c];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[q][c] = fmaf(bv[q], av[c], acc[q][c]);
   }
   uint32_t nan_count = 0;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const int64_t n = n0 + warp * 4 + q, b = b0 + lane + 32 * c;
+    for (int c = 0; c < 4; ++c) {
+      const int64_t n = n0 + ty * 4 + q, b = b0 + tx + 16 * c;
       if (n < N && b < G) {
         const int64_t i = n * G + b;
         const float L = fmaf(aor, acc[q][c], scale_value<FMT>(base[i], ws2));
@@ -278,99 +284,133 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
   if (nonfinite) warp_add_i32(nonfinite, nan_count);
 }
 
-// Adapter gradients from the masked scale gradient g [N, G]: dB[n,j] = (alpha/r) sum_b
-// g[n,b] A[j,b] and dA[j,b] = (alpha/r) sum_n B[n,j] g[n,b], fp32 accumulation in a fixed
-// order (the same result on every run).
-//
-// dB: one warp per row n, 32 j at a time; each lane sums over the columns b = lane
-// (mod 32) of 256-column chunks of A staged in shared memory, then a butterfly sums
-// the lanes.
-constexpr int kDbChunk = 256;
-constexpr int kWarps = kThreads / 32;
+// Adapter gradients from the masked scale gradient g [N, G], as two products with
+// the contraction split into chunks (one CTA per 64 x 64 output tile and chunk,
+// partial results summed by a second kernel in chunk order):
+//   dB[n,j] = (alpha/r) sum_b g[n,b] A[j,b]      (P = g, Q^T = A; contraction over b)
+//   dA[j,b] = (alpha/r) sum_n B[n,j] g[n,b]      (P = B^T, Q = g; contraction over n)
+// A CTA stages kKStep contraction indices of both operands per step in shared
+// memory (fp32), loading the next step into registers while it computes this one.
+constexpr int kKStep = 16;  // contraction indices per staged step
 
-__global__ void __launch_bounds__(kThreads) sq_lowrank_db_kernel(int64_t N, int64_t G, int r, float aor,
-                                                                 const float *__restrict__ g,
-                                                                 const uint16_t *__restrict__ A,
-                                                                 float *__restrict__ dB) {
-  extern __shared__ uint16_t db_smem[];  // [r][kDbChunk] chunk of A
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t n = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
-  for (int jc = 0; jc < r; jc += 32) {
-    const int nj = min(32, r - jc);
-    float acc[32];
+// Operand element (row i of the output, contraction index k) for the two products.
+struct DbLeft {  // g[n = i][b = k]
+  const float *g;
+  int64_t G;
+  __device__ float operator()(int64_t i, int64_t k) const { return g[i * G + k]; }
+};
+struct DbRight {  // A[j = i][b = k]
+  const uint16_t *A;
+  int64_t G;
+  __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(A[i * G + k]); }
+};
+struct DaLeft {  // B[n = k][j = i]
+  const uint16_t *B;
+  int r;
+  __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(B[k * r + i]); }
+};
+struct DaRight {  // g[n = k][b = i]
+  const float *g;
+  int64_t G;
+  __device__ float operator()(int64_t i, int64_t k) const { return g[k * G + i]; }
+};
+
+// partial[z][i][j] = sum_{k in chunk z} L(i, k) R(j, k), i < rows, j < cols.
+template <class LeftT, class RightT, bool LEFT_K_FAST, bool RIGHT_K_FAST>
+__global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t rows, int64_t cols, int64_t kdim,
+                                                                      int64_t kchunk, LeftT left, RightT right,
+                                                                      float *__restrict__ partial) {
+  __shared__ float sl[2][kKStep][kT + 1];  // [buffer][k][i]
+  __shared__ float sr[2][kKStep][kT + 1];  // [buffer][k][j]
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * kT;
+  const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kT;
+  const int64_t kb = static_cast<int64_t>(blockIdx.z) * kchunk;
+  const int64_t ke = kdim < kb + kchunk ? kdim : kb + kchunk;
+  const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+  // staging map: 4 elements of each operand per thread and step; consecutive threads
+  // walk the operand's contiguous index (k when it is the fast one, else the row)
+  float pl[4], pr[4];
+  auto load = [&](int64_t k0) {
 #pragma unroll
-    for (int t = 0; t < 32; ++t) acc[t] = 0.f;
-    for (int64_t bc = 0; bc < G; bc += kDbChunk) {
-      const int w = G - bc < kDbChunk ? static_cast<int>(G - bc) : kDbChunk;
-      __syncthreads();
-      for (int i = threadIdx.x; i < nj * kDbChunk; i += kThreads) {
-        const int t = i / kDbChunk, c = i % kDbChunk;
-        db_smem[i] = c < w ? A[static_cast<int64_t>(jc + t) * G + bc + c] : static_cast<uint16_t>(0);
-      }
-      __syncthreads();
-      if (n < N) {
-        for (int c = lane; c < w; c += 32) {
-          const float gv = g[n * G + bc + c];
-#pragma unroll
-          for (int t = 0; t < 32; ++t)
-            if (t < nj) acc[t] = fmaf(gv, bf16_bits(db_smem[t * kDbChunk + c]), acc[t]);
-        }
-      }
+    for (int e = 0; e < 4; ++e) {
+      const int idx = threadIdx.x + kThreads * e;  // 0 .. 1023 = kKStep * kT
+      const int kk_l = LEFT_K_FAST ? idx % kKStep : idx / kT, ii = LEFT_K_FAST ? idx / kKStep : idx % kT;
+      const int64_t k = k0 + kk_l, i = i0 + ii;
+      pl[e] = (k < ke && i < rows) ? left(i, k) : 0.f;
+      const int kk_r = RIGHT_K_FAST ? idx % kKStep : idx / kT, jj = RIGHT_K_FAST ? idx / kKStep : idx % kT;
+      const int64_t k2 = k0 + kk_r, j = j0 + jj;
+      pr[e] = (k2 < ke && j < cols) ? right(j, k2) : 0.f;
     }
+  };
+  auto store = [&](int buf) {
 #pragma unroll
-    for (int t = 0; t < 32; ++t) {
-      float v = acc[t];
+    for (int e = 0; e < 4; ++e) {
+      const int idx = threadIdx.x + kThreads * e;
+      const int kk_l = LEFT_K_FAST ? idx % kKStep : idx / kT, ii = LEFT_K_FAST ? idx / kKStep : idx % kT;
+      sl[buf][kk_l][ii] = pl[e];
+      const int kk_r = RIGHT_K_FAST ? idx % kKStep : idx / kT, jj = RIGHT_K_FAST ? idx / kKStep : idx % kT;
+      sr[buf][kk_r][jj] = pr[e];
+    }
+  };
+  float acc[4][4];
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-      if (n < N && lane == t && t < nj) dB[n * r + jc + t] = aor * v;
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[q][c] = 0.f;
+  int buf = 0;
+  load(kb);
+  store(0);
+  __syncthreads();
+  for (int64_t k0 = kb; k0 < ke; k0 += kKStep) {
+    const bool more = k0 + kKStep < ke;
+    if (more) load(k0 + kKStep);  // in flight while this step computes
+#pragma unroll
+    for (int kk = 0; kk < kKStep; ++kk) {
+      float lv[4], rv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) lv[q] = sl[buf][kk][ty * 4 + q];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) rv[c] = sr[buf][kk][tx + 16 * c];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[q][c] = fmaf(lv[q], rv[c], acc[q][c]);
+    }
+    if (more) {
+      store(buf ^ 1);
+      __syncthreads();
+      buf ^= 1;
     }
   }
+  float *out = partial + static_cast<int64_t>(blockIdx.z) * rows * cols;
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int64_t i = i0 + ty * 4 + q, j = j0 + tx + 16 * c;
+      if (i < rows && j < cols) out[i * cols + j] = acc[q][c];
+    }
 }
 
-// dA, pass 1: a CTA takes kDaRows rows n and 32 columns b; lane = column, warp w takes
-// j = w, w + 8, ...; the rows are summed in order into partial[chunk][j][b].
-constexpr int kDaRows = 128;
-constexpr int kDaJ = 32;  // accumulators per thread: r <= 8 * kDaJ = 256
-
-__global__ void __launch_bounds__(kThreads) sq_lowrank_da_partial_kernel(int64_t N, int64_t G, int r,
-                                                                         const float *__restrict__ g,
-                                                                         const uint16_t *__restrict__ B,
-                                                                         float *__restrict__ partial) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t chunk = blockIdx.x;
-  const int64_t b = static_cast<int64_t>(blockIdx.y) * 32 + lane;
-  const int64_t n0 = chunk * kDaRows, n1 = N < n0 + kDaRows ? N : n0 + kDaRows;
-  float acc[kDaJ];
-#pragma unroll
-  for (int t = 0; t < kDaJ; ++t) acc[t] = 0.f;
-  for (int64_t n = n0; n < n1; ++n) {
-    const float gv = b < G ? g[n * G + b] : 0.f;
-#pragma unroll
-    for (int t = 0; t < kDaJ; ++t) {
-      const int j = warp + kWarps * t;
-      if (j < r) acc[t] = fmaf(bf16_bits(B[n * r + j]), gv, acc[t]);
-    }
-  }
-  if (b < G) {
-#pragma unroll
-    for (int t = 0; t < kDaJ; ++t) {
-      const int j = warp + kWarps * t;
-      if (j < r) partial[(chunk * r + j) * G + b] = acc[t];
-    }
-  }
-}
-
-// dA, pass 2: dA[j,b] = (alpha/r) * sum over chunks, in chunk order.
-__global__ void __launch_bounds__(kThreads) sq_lowrank_da_reduce_kernel(int64_t G, int r, int64_t chunks, float aor,
-                                                                        const float *__restrict__ partial,
-                                                                        float *__restrict__ dA) {
-  const int64_t count = static_cast<int64_t>(r) * G;
+// out[i] = scale * sum over chunks z (in order) of partial[z][i].
+__global__ void __launch_bounds__(kThreads) sq_adapter_reduce_kernel(int64_t count, int64_t chunks, float scale,
+                                                                     const float *__restrict__ partial,
+                                                                     float *__restrict__ out) {
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < count;
        i += static_cast<int64_t>(gridDim.x) * kThreads) {
     float s = 0.f;
     for (int64_t c = 0; c < chunks; ++c) s += partial[c * count + i];
-    dA[i] = aor * s;
+    out[i] = scale * s;
   }
+}
+
+// Contraction chunks for an output of `tiles` 64 x 64 tiles: enough CTAs for about
+// two per SM, chunks of at least 4 steps.
+int64_t adapter_chunks(int64_t kdim, int64_t tiles, int sm_count) {
+  int64_t want = (2 * static_cast<int64_t>(sm_count) + tiles - 1) / tiles;
+  const int64_t most = (kdim + 4 * kKStep - 1) / (4 * kKStep);
+  if (want > most) want = most;
+  return want < 1 ? 1 : want;
 }
 
 unsigned grid_for(int64_t count, int sm_count) {
@@ -424,44 +464,63 @@ cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float w
     if (e != cudaSuccess) return e;
   }
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
-  const dim3 grid(static_cast<unsigned>((N + kLrRows - 1) / kLrRows), static_cast<unsigned>((G + kLrCols - 1) / kLrCols));
-  const size_t smem = static_cast<size_t>(kLrRows + kLrCols) * r * sizeof(uint16_t);
-  if (fmt == 0)
+  const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT));
+  const size_t smem = static_cast<size_t>(2 * kT) * r * sizeof(float);  // <= 128 KiB for r <= 256
+  cudaError_t e;
+  if (fmt == 0) {
+    if ((e = cudaFuncSetAttribute(sq_project_lowrank_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(smem))) != cudaSuccess)
+      return e;
     sq_project_lowrank_kernel<0><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
                                                                    bytes_out, mask_out, nonfinite, latent_out);
-  else
+  } else {
+    if ((e = cudaFuncSetAttribute(sq_project_lowrank_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(smem))) != cudaSuccess)
+      return e;
     sq_project_lowrank_kernel<1><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
                                                                    bytes_out, mask_out, nonfinite, latent_out);
+  }
   return cudaGetLastError();
 }
 
-size_t lowrank_grad_workspace(int64_t N, int64_t G, int r) {
-  const int64_t chunks = (N + kDaRows - 1) / kDaRows;
-  return static_cast<size_t>(chunks) * r * G * sizeof(float);
+// Workspace of the adapter gradients: the partial products of dB and of dA.
+size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count) {
+  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT), ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT);
+  const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);
+  return static_cast<size_t>(cb * N * r + ca * r * G) * sizeof(float);
 }
 
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
                                 cudaStream_t stream) {
-  if (dB) {
-    const unsigned grid = static_cast<unsigned>((N + kWarps - 1) / kWarps);
-    const size_t smem = static_cast<size_t>(min(r, 32)) * kDbChunk * sizeof(uint16_t);
-    sq_lowrank_db_kernel<<<grid, kThreads, smem, stream>>>(N, G, r, alpha_over_r, g, A, dB);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT), ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT);
+  const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);
+  float *pb = workspace, *pa = workspace + cb * N * r;
+  const unsigned reduce_cap = static_cast<unsigned>(sm_count) * kCtasPerSm;
+  cudaError_t e;
+  if (dB) {  // rows n, columns j, contraction b: g is b-contiguous, A is b-contiguous
+    const int64_t kc = ((G + cb - 1) / cb + kKStep - 1) / kKStep * kKStep;
+    const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((r + kT - 1) / kT),
+                    static_cast<unsigned>((G + kc - 1) / kc));
+    sq_adapter_product_kernel<DbLeft, DbRight, true, true><<<grid, kThreads, 0, stream>>>(
+        N, r, G, kc, DbLeft{g, G}, DbRight{A, G}, pb);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const int64_t count = N * r;
+    const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((count + kThreads - 1) / kThreads, reduce_cap));
+    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, grid.z, alpha_over_r, pb, dB);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  if (dA) {
-    const int64_t chunks = (N + kDaRows - 1) / kDaRows;
-    const dim3 grid1(static_cast<unsigned>(chunks), static_cast<unsigned>((G + 31) / 32));
-    sq_lowrank_da_partial_kernel<<<grid1, kThreads, 0, stream>>>(N, G, r, g, B, workspace);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+  if (dA) {  // rows j, columns b, contraction n: B is j-contiguous (row index fast), g is b-contiguous
+    const int64_t kc = ((N + ca - 1) / ca + kKStep - 1) / kKStep * kKStep;
+    const dim3 grid(static_cast<unsigned>((r + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT),
+                    static_cast<unsigned>((N + kc - 1) / kc));
+    sq_adapter_product_kernel<DaLeft, DaRight, false, false><<<grid, kThreads, 0, stream>>>(
+        r, G, N, kc, DaLeft{B, r}, DaRight{g, G}, pa);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int64_t count = static_cast<int64_t>(r) * G;
-    int64_t blocks = (count + kThreads - 1) / kThreads;
-    if (blocks > static_cast<int64_t>(sm_count) * kCtasPerSm) blocks = static_cast<int64_t>(sm_count) * kCtasPerSm;
-    sq_lowrank_da_reduce_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(G, r, chunks, alpha_over_r,
-                                                                                      workspace, dA);
-    return cudaGetLastError();
+    const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((count + kThreads - 1) / kThreads, reduce_cap));
+    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, grid.z, alpha_over_r, pa, dA);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
