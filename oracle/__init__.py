@@ -49,6 +49,10 @@ def lib():
         L.or_dx_at.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _i64, _p, _i64, _p, _p, _p]
         L.or_project.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
         L.or_merge.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p, _p]
+        L.or_rollback.argtypes = [ctypes.c_int, _i64, ctypes.c_float, _p, _p, _p]
+        L.or_swap.argtypes = [_i64, _p, _p, _p]
+        L.or_count_diff.restype = _i64
+        L.or_count_diff.argtypes = [_i64, _p, _p]
         L.or_lowrank_latent.restype = ctypes.c_float
         L.or_lowrank_latent.argtypes = [ctypes.c_int, ctypes.c_float, ctypes.c_float, ctypes.c_int, ctypes.c_uint8,
                                          _p, _p, _i64, _i64]
@@ -240,6 +244,36 @@ def merge(fmt, latent, scales, ws2, want_delta=True):
     ch = ctypes.c_int64(0)
     lib().or_merge(fmt, L.size, float(ws2), _ptr(L), _ptr(s), _ptr(delta), ctypes.byref(ch))
     return s, delta, int(ch.value)
+
+
+# --- rollback, hot-swap, audit (Sec. 5 Payoff 3, "Hot-swap") ----------------
+
+def rollback(fmt, scales, delta, ws2):
+    """Returns (restored bytes, changed): every byte replaced by the projection of
+    fl32(s(byte) - delta). `scales` is not modified."""
+    s = np.array(scales, dtype=np.uint8, copy=True, order="C")
+    d = _c(delta, np.float32)
+    assert d.shape == s.shape
+    ch = ctypes.c_int64(0)
+    lib().or_rollback(fmt, s.size, float(ws2), _ptr(d), _ptr(s), ctypes.byref(ch))
+    return s, int(ch.value)
+
+
+def swap(src, dst):
+    """Returns (new plane, changed): dst overwritten by src. `dst` is not modified."""
+    a = _c(src, np.uint8)
+    d = np.array(dst, dtype=np.uint8, copy=True, order="C")
+    assert a.shape == d.shape
+    ch = ctypes.c_int64(0)
+    lib().or_swap(a.size, _ptr(a), _ptr(d), ctypes.byref(ch))
+    return d, int(ch.value)
+
+
+def count_diff(a, b):
+    x = _c(a, np.uint8).reshape(-1)
+    y = _c(b, np.uint8).reshape(-1)
+    assert x.size == y.size
+    return int(lib().or_count_diff(x.size, _ptr(x), _ptr(y)))
 
 
 # --- low-rank scale adapter (Sec. 3 "Scale-QLoRA forward") -------------------

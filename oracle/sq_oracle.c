@@ -353,6 +353,43 @@ void or_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *s
     if (changed) *changed = ch;
 }
 
+/* Rollback (Sec. 5, Payoff 3: subtracting the on-grid scale delta the merge
+ * applied restores the base checkpoint byte for byte): every byte is replaced by
+ * the projection (same grid and clamp path as the merge) of fl32(s(byte) - delta)
+ * with s(byte) as or_scale_f32. changed = number of bytes that differ. */
+void or_rollback(int fmt, int64_t count, float ws2, const float *delta, uint8_t *scales_inout, int64_t *changed) {
+    int64_t ch = 0;
+    for (int64_t i = 0; i < count; i++) {
+        uint8_t b, mk;
+        int isn;
+        const uint8_t old = scales_inout[i];
+        const float back = or_scale_f32(fmt, ws2, old) - delta[i];
+        or_project_one(fmt, ws2, back, &b, &mk, &isn);
+        ch += (b != old);
+        scales_inout[i] = b;
+    }
+    if (changed) *changed = ch;
+}
+
+/* Scale-only hot-swap (Sec. 5 "Hot-swap"): the served task changes by overwriting
+ * the scale plane with another adapter's on-grid bytes; no code plane is an
+ * argument. changed = number of bytes that differ from the old plane. */
+void or_swap(int64_t count, const uint8_t *src, uint8_t *dst, int64_t *changed) {
+    int64_t ch = 0;
+    for (int64_t i = 0; i < count; i++) {
+        ch += (src[i] != dst[i]);
+        dst[i] = src[i];
+    }
+    if (changed) *changed = ch;
+}
+
+/* Byte-level audit (Sec. 5): the number of positions where two byte buffers differ. */
+int64_t or_count_diff(int64_t count, const uint8_t *a, const uint8_t *b) {
+    int64_t d = 0;
+    for (int64_t i = 0; i < count; i++) d += (a[i] != b[i]);
+    return d;
+}
+
 /* ------------------------------------------------------------------ */
 /* Low-rank scale adapter (Sec. 3 "Scale-QLoRA forward")                */
 /* ------------------------------------------------------------------ */
