@@ -11,6 +11,9 @@
  *   sq_merge           write on-grid bytes into the scale plane; never a code (Sec. 3, Sec. 5)
  *   sq_project_lowrank the low-rank adapter's latent eff + (alpha/r) B A, projected (Sec. 3)
  *   sq_lowrank_grad    gradients of the adapter factors B and A from the masked scale gradient
+ *   sq_rollback        undo a merge with its on-grid delta (Sec. 5 Payoff 3)
+ *   sq_swap_scales     scale-only hot-swap of the served adapter (Sec. 5)
+ *   sq_count_diff      byte-level audit of two buffers (Sec. 5)
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -133,6 +136,31 @@ sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, floa
  * changed_bytes device int64 or NULL: set to the number of bytes that changed. */
 sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
                    uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream);
+
+/* Rollback, Sec. 5 Payoff 3 ("invertible merges and rollback"): subtracting the
+ * on-grid scale delta a merge applied restores the base plane byte for byte. In
+ * place, every byte b of scales_inout becomes the projection (the merge's grid and
+ * clamp path) of fl32(s(b) - ongrid_delta), s(b) = fl32(E4M3(b) * ws2) or
+ * E8M0(b). The restoration is exact whenever each merged scale is within a factor
+ * 2 of its base (the subtraction is then exact in fp32); the raw training delta
+ * does not restore it. ongrid_delta device fp32 [N, G] (sq_merge's output);
+ * scales_inout device u8 [N, G]; changed_bytes device int64 or NULL (set). */
+sq_status sq_rollback(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *ongrid_delta,
+                      uint8_t *scales_inout, int64_t *changed_bytes, void *stream);
+
+/* Scale-only hot-swap, Sec. 5 "Hot-swap": the served task changes by overwriting
+ * the artifact's scale plane with another adapter's on-grid bytes; no code
+ * pointer is taken. src device u8 [N, G] (read); scales_inout device u8 [N, G]
+ * (overwritten); changed_bytes device int64 or NULL: set to the number of bytes
+ * that changed. */
+sq_status sq_swap_scales(sq_handle h, int64_t N, int64_t G, const uint8_t *src, uint8_t *scales_inout,
+                         int64_t *changed_bytes, void *stream);
+
+/* Byte-level audit (Sec. 5): *count (device int64, required) is set to the number
+ * of positions where the device buffers a and b (nbytes each, 16-byte aligned)
+ * differ, e.g. a code plane before and after a merge (expected 0). */
+sq_status sq_count_diff(sq_handle h, const uint8_t *a, const uint8_t *b, int64_t nbytes, int64_t *count,
+                        void *stream);
 
 /* Low-rank scale adapter, Sec. 3 "Scale-QLoRA forward": Delta S = (B A)(alpha/r)
  * with B [N, r] and A [r, G] (bf16 trainable factors), eff' = eff + Delta S per

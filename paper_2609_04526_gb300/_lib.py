@@ -27,7 +27,7 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 # Every entry point the header declares (checked against include/scaleqlora.h by the tests).
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
            "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
-           "sq_scale_grad_noalloc")
+           "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc")
 
 
 class SQError(RuntimeError):
@@ -69,6 +69,9 @@ def load() -> ctypes.CDLL:
     L.sq_merge.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
     L.sq_project_lowrank.argtypes = [vp, i32, i64, i64, i32, f32, f32, vp, vp, vp, vp, vp, vp, vp, vp]
     L.sq_lowrank_grad.argtypes = [vp, i64, i64, i32, f32, vp, vp, vp, vp, vp, vp]
+    L.sq_rollback.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp]
+    L.sq_swap_scales.argtypes = [vp, i64, i64, vp, vp, vp, vp]
+    L.sq_count_diff.argtypes = [vp, vp, vp, i64, vp, vp]
     L.sq_scale_grad_noalloc.argtypes = [W, vp, vp, i64, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
@@ -207,6 +210,31 @@ class Handle:
         self._check(self._L.sq_lowrank_grad(self._h, N, G, r, alpha_over_r, _ptr(g), _ptr(B), _ptr(A), _ptr(dB),
                                             _ptr(dA), _stream(stream)))
         return dB, dA
+
+    def sq_rollback(self, fmt: int, ongrid_delta: torch.Tensor, ws2: float, scales_inout: torch.Tensor,
+                    changed: Optional[torch.Tensor] = None, stream=None):
+        """Undo a merge in place with the on-grid delta it applied."""
+        N, G = scales_inout.shape
+        self._check(self._L.sq_rollback(self._h, fmt, N, G, ws2, _ptr(ongrid_delta), _ptr(scales_inout),
+                                        _ptr(changed), _stream(stream)))
+        return scales_inout
+
+    def sq_swap_scales(self, src: torch.Tensor, scales_inout: torch.Tensor, changed: Optional[torch.Tensor] = None,
+                       stream=None):
+        """Overwrite the scale plane with src (scale-only hot-swap), counting changed bytes."""
+        N, G = scales_inout.shape
+        self._check(self._L.sq_swap_scales(self._h, N, G, _ptr(src), _ptr(scales_inout), _ptr(changed),
+                                           _stream(stream)))
+        return scales_inout
+
+    def sq_count_diff(self, a: torch.Tensor, b: torch.Tensor, count: Optional[torch.Tensor] = None, stream=None):
+        """Device int64 tensor holding the number of differing bytes of a and b."""
+        if count is None:
+            count = torch.empty(1, dtype=torch.int64, device=a.device)
+        nbytes = a.numel() * a.element_size()
+        assert b.numel() * b.element_size() == nbytes
+        self._check(self._L.sq_count_diff(self._h, _ptr(a), _ptr(b), nbytes, _ptr(count), _stream(stream)))
+        return count
 
     def sq_merge(self, fmt: int, latent: torch.Tensor, ws2: float, scales_inout: torch.Tensor,
                  ongrid_delta: Optional[torch.Tensor] = None, changed: Optional[torch.Tensor] = None, stream=None):

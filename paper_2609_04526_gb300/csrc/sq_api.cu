@@ -378,6 +378,67 @@ sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, co
   SQ_GUARD_END
 }
 
+sq_status sq_rollback(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *ongrid_delta,
+                      uint8_t *scales_inout, int64_t *changed_bytes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_plane(h, fmt, N, G, ws2));
+  if (N * G > 0) {
+    SQ_TRY(check_buf(h, ongrid_delta, "ongrid_delta"));
+    SQ_TRY(check_buf(h, scales_inout, "scales_inout"));
+  }
+  if (changed_bytes && (reinterpret_cast<uintptr_t>(changed_bytes) & 7u))
+    return fail(h, SQ_ERR_INVALID_ARG, "changed_bytes must be 8-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_rollback(fmt, N * G, ws2, ongrid_delta, scales_inout, changed_bytes, dev->sm_count,
+                                       static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "rollback launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_swap_scales(sq_handle h, int64_t N, int64_t G, const uint8_t *src, uint8_t *scales_inout,
+                         int64_t *changed_bytes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  if (N * G > 0) {
+    SQ_TRY(check_buf(h, src, "src"));
+    SQ_TRY(check_buf(h, scales_inout, "scales_inout"));
+  }
+  if (changed_bytes && (reinterpret_cast<uintptr_t>(changed_bytes) & 7u))
+    return fail(h, SQ_ERR_INVALID_ARG, "changed_bytes must be 8-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_swap_or_diff(N * G, src, scales_inout, true, changed_bytes, dev->sm_count,
+                                           static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "swap launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_count_diff(sq_handle h, const uint8_t *a, const uint8_t *b, int64_t nbytes, int64_t *count,
+                        void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (nbytes < 0 || nbytes > (int64_t(1) << 40)) return fail(h, SQ_ERR_INVALID_ARG, "nbytes out of range");
+  if (nbytes > 0) {
+    SQ_TRY(check_buf(h, a, "a"));
+    SQ_TRY(check_buf(h, b, "b"));
+  }
+  if (!count || (reinterpret_cast<uintptr_t>(count) & 7u))
+    return fail(h, SQ_ERR_INVALID_ARG, "count must be non-NULL and 8-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_swap_or_diff(nbytes, a, const_cast<uint8_t *>(b), false, count, dev->sm_count,
+                                           static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "audit launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
 sq_status sq_project_lowrank(sq_handle h, int32_t fmt, int64_t N, int64_t G, int32_t r, float ws2, float alpha_over_r,
                              const uint8_t *base_scales, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
                              uint8_t *mask_out, int32_t *nonfinite, float *latent_out, void *stream) {

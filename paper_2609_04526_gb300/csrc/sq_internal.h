@@ -44,6 +44,13 @@ cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *laten
 cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *scales_inout,
                          float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream);
 
+// Rollback of a merge by its on-grid delta (in place, counting changed bytes), and
+// copy a -> b (write) or only count the bytes in which a and b differ.
+cudaError_t launch_rollback(int fmt, int64_t count, float ws2, const float *delta, uint8_t *scales_inout,
+                            int64_t *changed, int sm_count, cudaStream_t stream);
+cudaError_t launch_swap_or_diff(int64_t count, const uint8_t *a, uint8_t *b, bool write, int64_t *differing,
+                                int sm_count, cudaStream_t stream);
+
 // Low-rank scale adapter (Sec. 3 "Scale-QLoRA forward"): latent eff + (alpha/r) B A
 // projected onto the grid; and the gradients of B and A from the masked scale
 // gradient, through `workspace` (lowrank_grad_workspace bytes).

@@ -212,6 +212,85 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   if (changed) warp_add_i64(changed, n_changed);
 }
 
+// ---------------------------------------------------------------- rollback, swap, audit
+//
+// Sec. 5 Payoff 3: a merge is undone by subtracting the on-grid delta it applied;
+// each byte becomes the projection (the merge's grid and clamp path) of
+// fl32(s(byte) - delta). Sec. 5 "Hot-swap": the served task changes by overwriting
+// the scale plane with another adapter's bytes. Both count the bytes they change;
+// the audit counts the bytes in which two buffers differ (e.g. a code plane before
+// and after a merge). Same layout as the merge: 16 bytes per thread per step.
+
+__device__ __forceinline__ uint32_t bytes_differing(uint32_t a, uint32_t b) {
+  return static_cast<uint32_t>(__popc(__vcmpne4(a, b))) >> 3;  // 0xFF per differing byte
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_rollback_kernel(int64_t count, float ws2, float cap,
+                                                               const float *__restrict__ delta,
+                                                               uint8_t *__restrict__ scales,
+                                                               int64_t *__restrict__ changed) {
+  const int64_t nvec = count / 16;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  uint32_t n_changed = 0;
+  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    const float4 *src = reinterpret_cast<const float4 *>(delta) + 4 * v;
+    float d[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 f = __ldcs(src + q);
+      d[4 * q] = f.x;
+      d[4 * q + 1] = f.y;
+      d[4 * q + 2] = f.z;
+      d[4 * q + 3] = f.w;
+    }
+    const uint4 old4 = *(reinterpret_cast<const uint4 *>(scales) + v);
+    const uint32_t old[4] = {old4.x, old4.y, old4.z, old4.w};
+    uint32_t ob[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint32_t o = (old[i >> 2] >> (8 * (i & 3))) & 0xFFu;
+      uint32_t b, m, n;
+      project_one<FMT>(__fsub_rn(scale_value<FMT>(o, ws2), d[i]), ws2, cap, b, m, n);
+      ob[i >> 2] |= b << (8 * (i & 3));
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) n_changed += bytes_differing(ob[q], old[q]);
+    *(reinterpret_cast<uint4 *>(scales) + v) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
+    const int64_t i = nvec * 16 + threadIdx.x;
+    const uint32_t o = scales[i];
+    uint32_t b, m, n;
+    project_one<FMT>(__fsub_rn(scale_value<FMT>(o, ws2), delta[i]), ws2, cap, b, m, n);
+    scales[i] = static_cast<uint8_t>(b);
+    n_changed += (b != o) ? 1u : 0u;
+  }
+  if (changed) warp_add_i64(changed, n_changed);
+}
+
+// dst <- src (if src is non-null) and count the differing bytes of the two.
+__global__ void __launch_bounds__(kThreads) sq_swap_or_diff_kernel(int64_t count, const uint8_t *__restrict__ a,
+                                                                   uint8_t *__restrict__ b, bool write,
+                                                                   int64_t *__restrict__ differing) {
+  const int64_t nvec = count / 16;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  uint32_t n = 0;
+  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    const uint4 x = __ldcs(reinterpret_cast<const uint4 *>(a) + v);
+    const uint4 y = *(reinterpret_cast<const uint4 *>(b) + v);
+    n += bytes_differing(x.x, y.x) + bytes_differing(x.y, y.y) + bytes_differing(x.z, y.z) +
+         bytes_differing(x.w, y.w);
+    if (write) __stcs(reinterpret_cast<uint4 *>(b) + v, x);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
+    const int64_t i = nvec * 16 + threadIdx.x;
+    n += (a[i] != b[i]) ? 1u : 0u;
+    if (write) b[i] = a[i];
+  }
+  if (differing) warp_add_i64(differing, n);
+}
+
 // ---------------------------------------------------------------- low-rank scale adapter
 //
 // Sec. 3 "Scale-QLoRA forward": the latent block scale eff' = eff + (alpha/r) (B A),
@@ -523,6 +602,33 @@ cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r,
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+cudaError_t launch_rollback(int fmt, int64_t count, float ws2, const float *delta, uint8_t *scales_inout,
+                            int64_t *changed, int sm_count, cudaStream_t stream) {
+  if (changed) {
+    cudaError_t e = cudaMemsetAsync(changed, 0, sizeof(int64_t), stream);
+    if (e != cudaSuccess) return e;
+  }
+  if (count == 0) return cudaSuccess;
+  const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
+  const unsigned grid = grid_for(count, sm_count);
+  if (fmt == 0)
+    sq_rollback_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, delta, scales_inout, changed);
+  else
+    sq_rollback_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, delta, scales_inout, changed);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swap_or_diff(int64_t count, const uint8_t *a, uint8_t *b, bool write, int64_t *differing,
+                                int sm_count, cudaStream_t stream) {
+  if (differing) {
+    cudaError_t e = cudaMemsetAsync(differing, 0, sizeof(int64_t), stream);
+    if (e != cudaSuccess) return e;
+  }
+  if (count == 0) return cudaSuccess;
+  sq_swap_or_diff_kernel<<<grid_for(count, sm_count), kThreads, 0, stream>>>(count, a, b, write, differing);
+  return cudaGetLastError();
 }
 
 }  // namespace sqi
