@@ -347,10 +347,11 @@ PLANE_N, PLANE_G = 1 << 18, 1 << 10  # 2^28 scale blocks: far larger than the la
 
 
 def plane_ceiling(h, pk, stream, reps=10):
-    """Projection and merge over one synthetic 2^28-block NVFP4 plane: at the layer's
+    """The plane kernels over one synthetic 2^28-block NVFP4 plane: at the layer's
     sizes these launches last a few microseconds, so this shows their HBM ceiling.
     Bytes per block: projection 4 (latent) + 1 (byte) + 1 (mask); merge 4 + 1 (old
-    byte) + 1 (new byte)."""
+    byte) + 1 (new byte); rollback 4 (delta) + 1 + 1; swap 1 (source) + 1 + 1;
+    audit 1 + 1."""
     gen = torch.Generator(device="cuda").manual_seed(2028)
     ws2 = 1.0 / (6 * 448)
     L = torch.exp(torch.randn(PLANE_N, PLANE_G, device="cuda", generator=gen) * 2.0 - 3.0) * (448 * ws2 / 20)
@@ -361,9 +362,16 @@ def plane_ceiling(h, pk, stream, reps=10):
     changed = torch.zeros(1, dtype=torch.int64, device="cuda")
     blocks = PLANE_N * PLANE_G
     out = {"blocks": blocks, "shape": [PLANE_N, PLANE_G], "format": "nvfp4"}
-    for name, fn in (("project", lambda: h.sq_project_scales(0, L, ws2, bytes_out=qb, mask_out=mask,
-                                                               nonfinite=nonfinite, stream=stream)),
-                     ("merge", lambda: h.sq_merge(0, L, ws2, art, changed=changed, stream=stream))):
+    delta = torch.zeros(PLANE_N, PLANE_G, dtype=torch.float32, device="cuda")
+    other = torch.empty_like(qb)
+    count = torch.zeros(1, dtype=torch.int64, device="cuda")
+    legs = (("project", 6, lambda: h.sq_project_scales(0, L, ws2, bytes_out=qb, mask_out=mask,
+                                                      nonfinite=nonfinite, stream=stream)),
+            ("merge", 6, lambda: h.sq_merge(0, L, ws2, art, changed=changed, stream=stream)),
+            ("rollback", 6, lambda: h.sq_rollback(0, delta, ws2, art, changed=changed, stream=stream)),  # delta, old, new
+            ("swap", 3, lambda: h.sq_swap_scales(qb, other, changed=changed, stream=stream)),           # src, old, new
+            ("audit", 2, lambda: h.sq_count_diff(qb, art, count=count, stream=stream)))                # two planes
+    for name, per_block, fn in legs:
         for _ in range(3):
             fn()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -374,10 +382,11 @@ def plane_ceiling(h, pk, stream, reps=10):
         e1.record(stream)
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / reps
-        gbs = 6 * blocks / (ms / 1e3) / 1e9
-        out[name] = {"ms": ms, "bytes": 6 * blocks, "achieved": gbs, "unit": "GB/s", "frac": gbs / pk["hbm_gbs"]}
+        gbs = per_block * blocks / (ms / 1e3) / 1e9
+        out[name] = {"ms": ms, "bytes": per_block * blocks, "achieved": gbs, "unit": "GB/s",
+                     "frac": gbs / pk["hbm_gbs"]}
     h.sq_sync(stream)
-    del L, qb, mask, art
+    del L, qb, mask, art, delta, other
     return out
 
 

@@ -269,19 +269,40 @@ __global__ void __launch_bounds__(kThreads) sq_rollback_kernel(int64_t count, fl
   if (changed) warp_add_i64(changed, n_changed);
 }
 
-// dst <- src (if src is non-null) and count the differing bytes of the two.
+// b <- a (when `write`) and count the bytes in which a and b differ. A thread loads
+// four 16-byte vectors of each buffer before it stores any: a store to the address
+// just loaded waits for that load, so one vector per step would serialise every
+// thread on the memory latency.
+constexpr int kSwapUnroll = 4;
+
 __global__ void __launch_bounds__(kThreads) sq_swap_or_diff_kernel(int64_t count, const uint8_t *__restrict__ a,
                                                                    uint8_t *__restrict__ b, bool write,
                                                                    int64_t *__restrict__ differing) {
   const int64_t nvec = count / 16;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const uint4 *va = reinterpret_cast<const uint4 *>(a);
+  uint4 *vb = reinterpret_cast<uint4 *>(b);
   uint32_t n = 0;
-  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
-    const uint4 x = __ldcs(reinterpret_cast<const uint4 *>(a) + v);
-    const uint4 y = *(reinterpret_cast<const uint4 *>(b) + v);
-    n += bytes_differing(x.x, y.x) + bytes_differing(x.y, y.y) + bytes_differing(x.z, y.z) +
-         bytes_differing(x.w, y.w);
-    if (write) __stcs(reinterpret_cast<uint4 *>(b) + v, x);
+  for (int64_t v0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v0 < nvec;
+       v0 += stride * kSwapUnroll) {
+    uint4 x[kSwapUnroll], y[kSwapUnroll];
+#pragma unroll
+    for (int u = 0; u < kSwapUnroll; ++u) {
+      const int64_t v = v0 + stride * u;
+      if (v < nvec) {
+        x[u] = __ldcs(va + v);
+        y[u] = vb[v];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kSwapUnroll; ++u) {
+      const int64_t v = v0 + stride * u;
+      if (v < nvec) {
+        n += bytes_differing(x[u].x, y[u].x) + bytes_differing(x[u].y, y[u].y) + bytes_differing(x[u].z, y[u].z) +
+             bytes_differing(x[u].w, y[u].w);
+        if (write) __stcs(vb + v, x[u]);
+      }
+    }
   }
   if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
     const int64_t i = nvec * 16 + threadIdx.x;
