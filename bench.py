@@ -60,19 +60,20 @@ def parse_args():
 
 
 def profiled_traffic(workload):
-    """DRAM bytes per launch measured by ncu for each kernel kind (profiles/), or
-    None for every kind when the kernel sources changed since the capture."""
+    """DRAM bytes per launch measured by ncu for each kernel kind (profiles/); a kind
+    is left out when the source file of its kernel changed since the capture."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"traffic_{workload}_layer_step.json")
     if not os.path.exists(path):
         return {}
     with open(path) as f:
         prof = json.load(f)
-    for name, digest in prof.get("source_sha256", {}).items():
-        src = os.path.join(ROOT, "paper_2609_04526_gb300", "csrc", name)
-        if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != digest:
-            return {}
-    return prof.get("kernels", {})
+    out = {}
+    for kind, entry in prof.get("kernels", {}).items():
+        src = os.path.join(ROOT, "paper_2609_04526_gb300", "csrc", entry.get("source", ""))
+        if os.path.isfile(src) and hashlib.sha256(open(src, "rb").read()).hexdigest() == entry.get("source_sha256"):
+            out[kind] = entry
+    return out
 
 
 def peaks():
@@ -640,7 +641,7 @@ def run_ours(args):
                          "traffic": traffic.get(dom, {}).get("dram_bytes_per_launch"),
                          "algorithmic_bytes": traffic.get(dom, {}).get("algorithmic_bytes_per_launch"),
                          "traffic_note": "ncu dram bytes per launch, mean over the layer's 7 launches of this kernel "
-                                         "(profiles/traffic_c5_layer_step.json); null if the kernels changed since",
+                                         "(profiles/traffic_c5_layer_step.json); null if its source changed since",
                          "peak_source": f"{pk['source']} bf16 sustained"},
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels,
