@@ -14,6 +14,7 @@
  *   sq_rollback        undo a merge with its on-grid delta (Sec. 5 Payoff 3)
  *   sq_swap_scales     scale-only hot-swap of the served adapter (Sec. 5)
  *   sq_count_diff      byte-level audit of two buffers (Sec. 5)
+ *   sq_grouped_*       the three contractions over the experts of an MoE layer (Sec. 3)
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -218,6 +219,53 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
  * SQ_ERR_CUDA; there is no handle, so no error text. */
 sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
                                 const uint8_t *mask, float *g, int32_t *device_status, void *stream);
+
+/* ---------------------------------------------------------------- experts
+ * Mixture-of-experts layers (Sec. 3 "MoE: a batched grouped-expert kernel": the
+ * quantized linears are the experts, and every expert's contraction runs in one
+ * batched launch instead of a per-expert loop). One call covers the E experts of
+ * one linear; each expert e computes exactly what the dense entry point computes
+ * for its own weight and its own tokens.
+ *
+ * Token layout: the M = offsets[E] rows of X, dY, Y and dX are sorted by expert;
+ * rows offsets[e] .. offsets[e+1]-1 belong to expert e (a token routed to k
+ * experts appears k times). offsets is a HOST int64 array of E + 1 values with
+ * offsets[0] == 0, non-decreasing, offsets[E] < 2^31; an expert may have no rows.
+ *
+ * Each call builds a table of per-expert TMA descriptors in pinned host memory
+ * and copies it to the device on `stream` ahead of the kernel. The handle keeps
+ * four such tables per device and reuses them in turn: a call waits on the host
+ * until the grouped launch four calls back (on any stream) has completed. The
+ * host arrays (offsets, ws2) are read before the call returns. Grouped calls
+ * cannot be captured into a CUDA graph (SQ_ERR_UNSUPPORTED while the stream is
+ * capturing). */
+typedef struct {
+  int32_t fmt;           /* sq_format, shared by all experts                            */
+  int32_t E;             /* experts, 1 <= E <= 65536, with E * N <= 2^31 - 1025         */
+  int32_t N;             /* out features of each expert, N % 8 == 0                     */
+  int32_t K;             /* in features of each expert,  K % 32 == 0                    */
+  const uint8_t *codes;  /* device [E, N, K/2]: expert e's codes at e * N * K/2 bytes   */
+  const uint8_t *scales; /* device [E, N, K/B]: expert e's scale plane                  */
+  const float *ws2;      /* HOST [E]: NVFP4 tensor scale of each expert (finite, > 0);
+                            MXFP4: NULL, or every entry exactly 1.0                     */
+} sq_grouped_weight;
+
+/* Y[offsets[e] + m, :] = X[offsets[e] + m, :] . W_e^T for every expert e.
+ * X device bf16 [M, K]; Y device bf16 [M, N]. M == 0 writes nothing. */
+sq_status sq_grouped_fwd(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
+                         uint16_t *Y, void *stream);
+
+/* dX[offsets[e] + m, :] = dY[offsets[e] + m, :] . W_e for every expert e.
+ * dY device bf16 [M, N]; dX device bf16 [M, K]. */
+sq_status sq_grouped_bwd_dx(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *dY,
+                            uint16_t *dX, void *stream);
+
+/* g[e, n, b] = sum_{k in b} code_e[n, k] sum over expert e's rows m of dY[m, n] X[m, k]
+ * (optionally x mask[e, n, b]); an expert with no rows gets g[e] = 0.
+ * X device bf16 [M, K]; dY device bf16 [M, N]; mask device u8 [E, N, K/B] or NULL;
+ * g device fp32 [E, N, K/B]. The scale bytes are not read (scales may be NULL). */
+sq_status sq_grouped_scale_grad(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
+                                const uint16_t *dY, const uint8_t *mask, float *g, void *stream);
 
 #ifdef __cplusplus
 }

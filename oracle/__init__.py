@@ -311,3 +311,49 @@ def lowrank_grad(gm, B_bits, A_bits, alpha_over_r):
     dA = np.empty((r, G), dtype=np.float64)
     lib().or_lowrank_grad(N, G, r, float(alpha_over_r), _ptr(g), _ptr(B), _ptr(A), _ptr(dB), _ptr(dA))
     return dB, dA
+
+
+# --- experts of an MoE linear (Sec. 3 "MoE: a batched grouped-expert kernel") -
+# The quantized linears of an MoE layer are its experts: expert e owns the token
+# rows offsets[e] .. offsets[e+1]-1 (sorted by expert) and computes, on those rows
+# alone, exactly the dense step above with its own codes, scales and ws2.
+
+def _expert_rows(offsets, e):
+    return int(offsets[e]), int(offsets[e + 1])
+
+
+def grouped_fwd(fmt, codes, scales, ws2, offsets, X_bits):
+    """Y [M, N]: the forward of expert e on its rows, for every e.
+    codes [E, N, K/2], scales [E, N, G] u8; ws2 one value per expert."""
+    E, N = codes.shape[0], codes.shape[1]
+    Y = np.zeros((int(offsets[E]), N), dtype=np.float64)
+    for e in range(E):
+        a, b = _expert_rows(offsets, e)
+        if b > a:
+            Y[a:b] = fwd(fmt, codes[e], scales[e], ws2[e], X_bits[a:b])
+    return Y
+
+
+def grouped_dx(fmt, codes, scales, ws2, offsets, dY_bits):
+    """dX [M, K]: the input gradient of expert e on its rows, for every e."""
+    E, K = codes.shape[0], codes.shape[2] * 2
+    dX = np.zeros((int(offsets[E]), K), dtype=np.float64)
+    for e in range(E):
+        a, b = _expert_rows(offsets, e)
+        if b > a:
+            dX[a:b] = dx(fmt, codes[e], scales[e], ws2[e], dY_bits[a:b])
+    return dX
+
+
+def grouped_scale_grad(fmt, codes, offsets, X_bits, dY_bits, mask=None, experts=None):
+    """g [E, N, G]: expert e's block-reduced scale gradient over its own rows (zero
+    for an expert without rows), optionally times mask [E, N, G]. `experts` limits
+    the work to those experts (the others are left zero)."""
+    E, N, K = codes.shape[0], codes.shape[1], codes.shape[2] * 2
+    G = K // BLOCK[fmt]
+    g = np.zeros((E, N, G), dtype=np.float64)
+    for e in (range(E) if experts is None else experts):
+        a, b = _expert_rows(offsets, e)
+        if b > a:
+            g[e] = scale_grad(fmt, codes[e], X_bits[a:b], dY_bits[a:b], None if mask is None else mask[e])
+    return g

@@ -4,4 +4,4 @@ The compute lives in libscaleqlora.so (C ABI in include/scaleqlora.h); this
 package holds its ctypes binding (`_lib`), the nvcc build (`build`) and the
 seeded synthetic-workload generator (`synth`).
 """
-from ._lib import BLOCK, MXFP4, NVFP4, Handle, QuantWeight, SQError, load  # noqa: F401
+from ._lib import BLOCK, MXFP4, NVFP4, GroupedWeight, Handle, QuantWeight, SQError, load  # noqa: F401

@@ -27,7 +27,8 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 # Every entry point the header declares (checked against include/scaleqlora.h by the tests).
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
            "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
-           "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc")
+           "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
+           "sq_grouped_bwd_dx", "sq_grouped_scale_grad")
 
 
 class SQError(RuntimeError):
@@ -39,6 +40,11 @@ class SQError(RuntimeError):
 class _SqWeight(ctypes.Structure):
     _fields_ = [("fmt", ctypes.c_int32), ("N", ctypes.c_int32), ("K", ctypes.c_int32),
                 ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("ws2", ctypes.c_float)]
+
+
+class _SqGroupedWeight(ctypes.Structure):
+    _fields_ = [("fmt", ctypes.c_int32), ("E", ctypes.c_int32), ("N", ctypes.c_int32), ("K", ctypes.c_int32),
+                ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("ws2", ctypes.POINTER(ctypes.c_float))]
 
 
 _lib = None
@@ -73,6 +79,10 @@ def load() -> ctypes.CDLL:
     L.sq_swap_scales.argtypes = [vp, i64, i64, vp, vp, vp, vp]
     L.sq_count_diff.argtypes = [vp, vp, vp, i64, vp, vp]
     L.sq_scale_grad_noalloc.argtypes = [W, vp, vp, i64, vp, vp, vp, vp]
+    GW, OFF = ctypes.POINTER(_SqGroupedWeight), ctypes.POINTER(ctypes.c_int64)
+    L.sq_grouped_fwd.argtypes = [vp, GW, OFF, vp, vp, vp]
+    L.sq_grouped_bwd_dx.argtypes = [vp, GW, OFF, vp, vp, vp]
+    L.sq_grouped_scale_grad.argtypes = [vp, GW, OFF, vp, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
@@ -92,6 +102,37 @@ class QuantWeight:
 
     def _c(self) -> _SqWeight:
         return _SqWeight(self.fmt, self.N, self.K, _ptr(self.codes), _ptr(self.scales), self.ws2)
+
+
+@dataclasses.dataclass
+class GroupedWeight:
+    """The E experts of one MoE linear, each [N, K]: codes [E, N, K/2] u8, scales
+    [E, N, K/B] u8 (device), ws2 one tensor scale per expert (host floats)."""
+    fmt: int
+    E: int
+    N: int
+    K: int
+    codes: torch.Tensor
+    scales: Optional[torch.Tensor]
+    ws2: list
+
+    def _c(self):
+        ws = (ctypes.c_float * self.E)(*[float(x) for x in self.ws2])
+        c = _SqGroupedWeight(self.fmt, self.E, self.N, self.K, _ptr(self.codes), _ptr(self.scales),
+                             ctypes.cast(ws, ctypes.POINTER(ctypes.c_float)))
+        return c, ws  # keep the array alive for the call
+
+    def expert(self, e: int) -> QuantWeight:
+        """Expert e as a dense weight (views into the grouped planes)."""
+        return QuantWeight(self.fmt, self.N, self.K, self.codes[e],
+                           None if self.scales is None else self.scales[e], float(self.ws2[e]))
+
+
+def _offsets(offsets, E: int):
+    vals = [int(x) for x in offsets]
+    if len(vals) != E + 1:  # the library reads exactly E + 1 values
+        raise ValueError(f"offsets has {len(vals)} values; a grouped call over {E} experts needs {E + 1}")
+    return (ctypes.c_int64 * len(vals))(*vals), vals
 
 
 def _ptr(t: Optional[torch.Tensor]):
@@ -242,3 +283,34 @@ class Handle:
         self._check(self._L.sq_merge(self._h, fmt, N, G, ws2, _ptr(latent), _ptr(scales_inout), _ptr(ongrid_delta),
                                      _ptr(changed), _stream(stream)))
         return scales_inout
+
+    # experts of an MoE linear ------------------------------------------------
+    def sq_grouped_fwd(self, w: GroupedWeight, offsets, X: torch.Tensor, Y: Optional[torch.Tensor] = None,
+                       stream=None):
+        """Y rows offsets[e]..offsets[e+1]-1 = X rows of expert e times W_e^T (offsets: E + 1 host ints)."""
+        off, vals = _offsets(offsets, w.E)
+        if Y is None:
+            Y = torch.empty(vals[-1], w.N, dtype=torch.bfloat16, device=X.device)
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_fwd(self._h, ctypes.byref(wc), off, _ptr(X), _ptr(Y), _stream(stream)))
+        return Y
+
+    def sq_grouped_bwd_dx(self, w: GroupedWeight, offsets, dY: torch.Tensor, dX: Optional[torch.Tensor] = None,
+                          stream=None):
+        off, vals = _offsets(offsets, w.E)
+        if dX is None:
+            dX = torch.empty(vals[-1], w.K, dtype=torch.bfloat16, device=dY.device)
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_bwd_dx(self._h, ctypes.byref(wc), off, _ptr(dY), _ptr(dX), _stream(stream)))
+        return dX
+
+    def sq_grouped_scale_grad(self, w: GroupedWeight, offsets, X: torch.Tensor, dY: torch.Tensor,
+                              mask: Optional[torch.Tensor] = None, g: Optional[torch.Tensor] = None, stream=None):
+        """g [E, N, K/B] fp32: every expert's block-reduced scale gradient over its own rows."""
+        off, _ = _offsets(offsets, w.E)
+        if g is None:
+            g = torch.empty(w.E, w.N, w.K // BLOCK[w.fmt], dtype=torch.float32, device=X.device)
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_scale_grad(self._h, ctypes.byref(wc), off, _ptr(X), _ptr(dY), _ptr(mask),
+                                                  _ptr(g), _stream(stream)))
+        return g

@@ -19,12 +19,26 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// One expert table of a grouped launch: built in pinned host memory, copied to
+// the device on the call's stream. `done` is recorded after the launch that reads
+// it, so the slot is rewritten only once that launch (and its copy) completed.
+struct TableSlot {
+  uint8_t *host = nullptr;
+  uint8_t *dev = nullptr;
+  size_t bytes = 0;
+  cudaEvent_t done = nullptr;
+  bool pending = false;
+};
+constexpr int kTableSlots = 4;
+
 struct DeviceState {
   int device;
   int sm_count;
   int *err_word;         // device int, written by kernels whose bounded waits ran out
   void *workspace;       // scratch of the adapter-gradient kernels, grown on demand
   size_t workspace_bytes;
+  TableSlot tables[kTableSlots];
+  int next_table;
 };
 
 constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
@@ -87,7 +101,7 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   int *err_word = nullptr;
   if ((e = cudaMalloc(&err_word, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(error word)");
   if ((e = cudaMemset(err_word, 0, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(error word)");
-  h->devices.push_back(DeviceState{dev, sms, err_word, nullptr, 0});
+  h->devices.push_back(DeviceState{dev, sms, err_word, nullptr, 0, {}, 0});
   *out = &h->devices.back();
   return SQ_OK;
 }
@@ -209,6 +223,166 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   return SQ_OK;
 }
 
+// ------------------------------------------------------------------ grouped (experts)
+
+constexpr int kMaxExperts = 1 << 16;
+
+// Shape, scale and token-layout checks of a grouped call; on success `rows`
+// holds each expert's token count and M the total.
+sq_status check_grouped(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, bool need_scales,
+                        std::vector<int64_t> &rows, int64_t &M) {
+  if (!w) return fail(h, SQ_ERR_INVALID_ARG, "grouped weight is NULL");
+  if (w->E < 1 || w->E > kMaxExperts) return fail(h, SQ_ERR_INVALID_ARG, "E=%d must be in [1, 65536]", w->E);
+  if (w->fmt != SQ_NVFP4 && w->fmt != SQ_MXFP4) return fail(h, SQ_ERR_INVALID_ARG, "unknown format %d", w->fmt);
+  for (int e = 0; e < w->E; ++e) {
+    const float ws2 = w->ws2 ? w->ws2[e] : 1.0f;
+    if (w->fmt == SQ_NVFP4 && !w->ws2) return fail(h, SQ_ERR_INVALID_ARG, "NVFP4 experts need ws2[E]");
+    if (w->fmt == SQ_NVFP4 && !(std::isfinite(ws2) && ws2 > 0.0f))
+      return fail(h, SQ_ERR_INVALID_ARG, "ws2[%d] must be finite and > 0", e);
+    if (w->fmt == SQ_MXFP4 && ws2 != 1.0f) return fail(h, SQ_ERR_INVALID_ARG, "MXFP4 ws2[%d] must be 1.0", e);
+  }
+  if (w->N <= 0 || w->N % 8 != 0 || w->N > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "N=%d must be positive, a multiple of 8 and <= 2^24", w->N);
+  if (w->K <= 0 || w->K % 32 != 0 || w->K > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "K=%d must be positive, a multiple of 32 and <= 2^24", w->K);
+  // code rows of all experts are addressed with int32 TMA coordinates (plus one tile of overhang)
+  if (static_cast<int64_t>(w->E) * w->N + 1024 > kMaxTokens)
+    return fail(h, SQ_ERR_INVALID_ARG, "E * N = %lld code rows exceed 2^31 - 1024", (long long)w->E * w->N);
+  if (!w->codes || !aligned16(w->codes)) return fail(h, SQ_ERR_INVALID_ARG, "codes must be non-NULL and 16-byte aligned");
+  if (need_scales && (!w->scales || !aligned16(w->scales)))
+    return fail(h, SQ_ERR_INVALID_ARG, "scales must be non-NULL and 16-byte aligned");
+  if (!offsets) return fail(h, SQ_ERR_INVALID_ARG, "offsets is NULL");
+  if (offsets[0] != 0) return fail(h, SQ_ERR_INVALID_ARG, "offsets[0] must be 0");
+  rows.assign(w->E, 0);
+  for (int e = 0; e < w->E; ++e) {
+    if (offsets[e + 1] < offsets[e])
+      return fail(h, SQ_ERR_INVALID_ARG, "offsets must be non-decreasing (offsets[%d] < offsets[%d])", e + 1, e);
+    rows[e] = offsets[e + 1] - offsets[e];
+  }
+  M = offsets[w->E];
+  return check_tokens(h, M);
+}
+
+// The next expert-table slot of the device, at least `bytes` large. Waits on the
+// host for the launch that last read the slot (kTableSlots grouped calls back).
+sq_status acquire_table(sq_handle h, DeviceState *dev, size_t bytes, TableSlot **out) {
+  TableSlot &t = dev->tables[dev->next_table];
+  dev->next_table = (dev->next_table + 1) % kTableSlots;
+  cudaError_t e;
+  if (!t.done && (e = cudaEventCreateWithFlags(&t.done, cudaEventDisableTiming)) != cudaSuccess)
+    return cuda_fail(h, e, "cudaEventCreate(table)");
+  if (t.pending) {
+    if ((e = cudaEventSynchronize(t.done)) != cudaSuccess) return cuda_fail(h, e, "waiting for an expert table");
+    t.pending = false;
+  }
+  if (bytes > t.bytes) {
+    if (t.dev) cudaFree(t.dev);
+    if (t.host) cudaFreeHost(t.host);
+    t.dev = t.host = nullptr;
+    t.bytes = 0;
+    const size_t cap = (bytes + 65535) & ~size_t(65535);
+    if ((e = cudaMalloc(&t.dev, cap)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(expert table)");
+    if ((e = cudaMallocHost(&t.host, cap)) != cudaSuccess) return cuda_fail(h, e, "cudaMallocHost(expert table)");
+    t.bytes = cap;
+  }
+  *out = &t;
+  return SQ_OK;
+}
+
+// One grouped contraction. FWD: a = X [M, K], out = Y [M, N]. DX: a = dY [M, N],
+// out = dX [M, K]. SGRAD: a = dY, b = X, out = g [E, N, G].
+sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const std::vector<int64_t> &rows,
+                      const int64_t *offsets, const uint16_t *a_ptr, const uint16_t *b_ptr, void *out,
+                      const uint8_t *mask, cudaStream_t stream) {
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(stream, &cap);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
+  if (cap != cudaStreamCaptureStatusNone)
+    return fail(h, SQ_ERR_UNSUPPORTED, "grouped calls copy a host-built expert table and cannot be graph-captured");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const int E = w->E;
+  const int64_t N = w->N, K = w->K;
+  // the tile list: FWD / DX ceil(M_e / 512) row tiles of each expert x its column
+  // tiles; SGRAD every expert's full (N / 256) x (K / 256) grid, empty experts included
+  std::vector<int32_t> tile_start(E + 1, 0);
+  int64_t total = 0;
+  if (mode == sqi::MODE_SGRAD) {
+    const int64_t per = ((N + sqi::kSgradTile - 1) / sqi::kSgradTile) * ((K + sqi::kSgradTile - 1) / sqi::kSgradTile);
+    for (int x = 0; x < E; ++x) {
+      tile_start[x] = static_cast<int32_t>(total);
+      total += per;
+      if (total > kMaxTokens) return fail(h, SQ_ERR_INVALID_ARG, "too many tiles");
+    }
+  } else {
+    const int64_t tn = ((mode == sqi::MODE_FWD ? N : K) + sqi::kPairNTile - 1) / sqi::kPairNTile;
+    for (int x = 0; x < E; ++x) {
+      tile_start[x] = static_cast<int32_t>(total);
+      total += (rows[x] + sqi::kPairMTile - 1) / sqi::kPairMTile * tn;
+      if (total > kMaxTokens) return fail(h, SQ_ERR_INVALID_ARG, "too many tiles");
+    }
+  }
+  tile_start[E] = static_cast<int32_t>(total);
+  if (total == 0) return SQ_OK;
+
+  TableSlot *t = nullptr;
+  const size_t bytes = sqi::group_table_bytes(E);
+  SQ_TRY(acquire_table(h, dev, bytes, &t));
+  std::memset(t->host, 0, bytes);
+  auto *maps = reinterpret_cast<sqi::GroupMaps *>(t->host);
+  for (int x = 0; x < E; ++x) {
+    if (rows[x] == 0) continue;  // no tiles read this expert's descriptors
+    const int64_t m = rows[x], r0 = offsets[x];
+    if (mode == sqi::MODE_FWD) {
+      SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * K, K, m, 64, sqi::kBM));
+      SQ_TRY(make_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * N, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                      N, m, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B));
+    } else if (mode == sqi::MODE_DX) {
+      SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * N, N, m, 64, sqi::kBM));
+      SQ_TRY(make_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * K, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                      K, m, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B));
+    } else {
+      SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * N, N, m, 64, sqi::kSgradBK));
+      SQ_TRY(make_act_map(h, &maps[x].m[1], b_ptr + r0 * K, K, m, 64, sqi::kSgradBK));
+    }
+  }
+  auto *ts = reinterpret_cast<int32_t *>(t->host + sqi::group_off_tiles(E));
+  auto *rw = reinterpret_cast<int32_t *>(t->host + sqi::group_off_rows(E));
+  auto *ws = reinterpret_cast<float *>(t->host + sqi::group_off_ws2(E));
+  for (int x = 0; x <= E; ++x) ts[x] = tile_start[x];
+  for (int x = 0; x < E; ++x) {
+    rw[x] = static_cast<int32_t>(rows[x]);
+    ws[x] = w->ws2 ? w->ws2[x] : 1.0f;
+  }
+  // all experts' codes as one [E * N, K/2] tensor, the dense kernels' code boxes
+  CUtensorMap tmCodes;
+  SQ_TRY(make_map(h, &tmCodes, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K / 2, static_cast<int64_t>(E) * N, 64,
+                  128, CU_TENSOR_MAP_SWIZZLE_64B));
+  if ((e = cudaMemcpyAsync(t->dev, t->host, bytes, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+    return cuda_fail(h, e, "copying the expert table");
+  sqi::GroupedArgs ga;
+  ga.mode = mode;
+  ga.fmt = w->fmt;
+  ga.E = E;
+  ga.N = N;
+  ga.K = K;
+  ga.codes = w->codes;
+  ga.scales = w->scales;
+  ga.out = out;
+  ga.mask = mask;
+  ga.err = dev->err_word;
+  ga.table = t->dev;
+  ga.total_tiles = static_cast<int>(total);
+  e = sqi::launch_grouped(ga, tmCodes, dev->sm_count, stream);
+  // the slot is busy until the copy and the kernel complete (recorded even after a
+  // failed launch, so the slot's next user waits only for the copy)
+  cudaError_t e2 = cudaEventRecord(t->done, stream);
+  if (e2 == cudaSuccess) t->pending = true;
+  if (e != cudaSuccess) return cuda_fail(h, e, "grouped kernel launch");
+  if (e2 != cudaSuccess) return cuda_fail(h, e2, "cudaEventRecord(table)");
+  return SQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -232,6 +406,14 @@ sq_status sq_destroy(sq_handle h) {
     if (cudaSetDevice(d.device) == cudaSuccess) {
       cudaFree(d.err_word);
       if (d.workspace) cudaFree(d.workspace);
+      for (auto &t : d.tables) {
+        if (t.done) {
+          cudaEventSynchronize(t.done);
+          cudaEventDestroy(t.done);
+        }
+        if (t.dev) cudaFree(t.dev);
+        if (t.host) cudaFreeHost(t.host);
+      }
     }
   }
   if (cur >= 0) cudaSetDevice(cur);
@@ -502,6 +684,57 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
                                dev->sm_count, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");
   return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_fwd(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
+                         uint16_t *Y, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  std::vector<int64_t> rows;
+  int64_t M = 0;
+  SQ_TRY(check_grouped(h, w, offsets, true, rows, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, Y, "Y"));
+  return run_grouped(h, sqi::MODE_FWD, w, rows, offsets, X, nullptr, Y, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_bwd_dx(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *dY,
+                            uint16_t *dX, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  std::vector<int64_t> rows;
+  int64_t M = 0;
+  SQ_TRY(check_grouped(h, w, offsets, true, rows, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, dY, "dY"));
+  SQ_TRY(check_buf(h, dX, "dX"));
+  return run_grouped(h, sqi::MODE_DX, w, rows, offsets, dY, nullptr, dX, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_scale_grad(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
+                                const uint16_t *dY, const uint8_t *mask, float *g, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  std::vector<int64_t> rows;
+  int64_t M = 0;
+  SQ_TRY(check_grouped(h, w, offsets, false, rows, M));
+  SQ_TRY(check_buf(h, g, "g"));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (M == 0) {  // every sum is empty
+    DeviceState *dev = nullptr;
+    SQ_TRY(ensure_device(h, &dev));
+    const size_t bytes = static_cast<size_t>(w->E) * w->N * (w->K / block_of(w->fmt)) * sizeof(float);
+    cudaError_t e = cudaMemsetAsync(g, 0, bytes, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(g)");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, dY, "dY"));
+  return run_grouped(h, sqi::MODE_SGRAD, w, rows, offsets, dY, X, g, mask, st);
   SQ_GUARD_END
 }
 

@@ -31,6 +31,47 @@ struct GemmArgs {
   int *err;              // device error word
 };
 
+// Expert table of a grouped launch, built by the host for each call and copied
+// to the device ahead of the kernel (64-byte aligned):
+//   GroupMaps[E]         two TMA descriptors per expert, each addressing only that
+//                        expert's token rows: FWD / DX the streamed activations and
+//                        the output; SGRAD dY and X
+//   int32 tile_start[E+1] first tile of each expert in the launch's tile list
+//   int32 rows[E]        the expert's token count M_e
+//   float ws2[E]         the expert's tensor scale (1.0 for MXFP4)
+struct GroupMaps {
+  CUtensorMap m[2];
+};
+static_assert(sizeof(GroupMaps) == 256, "two 128-byte tensor maps per expert");
+__host__ __device__ constexpr size_t group_off_tiles(int E) { return static_cast<size_t>(E) * sizeof(GroupMaps); }
+__host__ __device__ constexpr size_t group_off_rows(int E) { return group_off_tiles(E) + static_cast<size_t>(E + 1) * 4; }
+__host__ __device__ constexpr size_t group_off_ws2(int E) { return group_off_rows(E) + static_cast<size_t>(E) * 4; }
+__host__ __device__ constexpr size_t group_table_bytes(int E) { return group_off_ws2(E) + static_cast<size_t>(E) * 4; }
+
+// Output rows of one FWD / DX tile and tokens of one scale-gradient stage: the
+// host sizes the grouped tile list with these.
+constexpr int kPairMTile = 512;
+constexpr int kPairNTile = 256;
+constexpr int kSgradTile = 256;
+
+struct GroupedArgs {
+  int mode;
+  int fmt;
+  int E;                 // experts
+  int64_t N, K;          // per expert: out features, in features
+  const uint8_t *codes;  // [E, N, K/2]
+  const uint8_t *scales; // [E, N, K/B]
+  void *out;             // MODE_SGRAD: g [E, N, K/B] f32 (FWD / DX write through the table's maps)
+  const uint8_t *mask;   // [E, N, K/B] or null (MODE_SGRAD only)
+  int *err;
+  const uint8_t *table;  // device copy of the expert table
+  int total_tiles;       // tile_start[E]
+};
+
+// Launch one grouped contraction. tmCodes is the descriptor of all experts'
+// packed codes as one [E * N, K/2] tensor (MODE_FWD / MODE_DX; unused for MODE_SGRAD).
+cudaError_t launch_grouped(const GroupedArgs &a, const CUtensorMap &tmCodes, int sm_count, cudaStream_t stream);
+
 // Launch one contraction. tmA is the TMA descriptor of the streamed bf16
 // activations; tmB that of the packed codes (MODE_FWD / MODE_DX) or of the second
 // bf16 operand (MODE_SGRAD); tmOut that of the bf16 output (MODE_FWD / MODE_DX:

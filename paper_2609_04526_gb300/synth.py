@@ -242,3 +242,109 @@ def gen_adapter(wl: Workload, lin: Linear, weight: Weight, r: int = 58, alpha: f
 
 def act_names(wl: Workload) -> List[str]:
     return [a[0] for a in wl.acts]
+
+
+# ---------------------------------------------------------------- MoE experts
+# The paper's MoE bases (Sec. 4: Qwen3-30B-A3B NVFP4; gpt-oss-120B, 128 experts,
+# native MXFP4) are not available offline and the paper prints no expert shapes;
+# these workloads take the experts' shapes from the public model configurations
+# (Qwen3-30B-A3B: 128 experts, top-8, hidden 2048, expert intermediate 768;
+# gpt-oss-120B: 128 experts, top-4, hidden 2880, intermediate 2880, its fused
+# gate/up projection drawn as two linears). A batch of T tokens is routed top-k
+# by a seeded router whose expert popularity is log-normal (route_sigma), so the
+# per-expert token counts are ragged like a load-balanced router's; tokens are
+# sorted by expert, so expert e owns rows offsets[e] .. offsets[e+1]-1.
+
+@dataclasses.dataclass(frozen=True)
+class MoEWorkload:
+    key: str
+    title: str
+    fmt: int
+    T: int                      # tokens of the batch
+    top_k: int                  # experts per token
+    E: int                      # experts per linear
+    linears: tuple              # per-expert Linear shapes
+    acts: tuple                 # (name, K, kind) as in Workload
+    seed: int
+    route_sigma: float = 0.3    # log-normal spread of the experts' popularity (max load ~2.2x the mean)
+    counts: Optional[tuple] = None  # fixed per-expert token counts (tests); else drawn by the router
+    w_std: float = 0.02
+    dy_std: float = 1e-3
+
+    @property
+    def block(self) -> int:
+        return BLOCK[self.fmt]
+
+    @property
+    def M(self) -> int:
+        """Routed token rows of every expert linear (each token appears top_k times)."""
+        return sum(self.counts) if self.counts is not None else self.T * self.top_k
+
+    def flops(self) -> int:
+        """6 * (routed rows) * N * K summed over the expert linears."""
+        return sum(6 * self.M * l.N * l.K for l in self.linears)
+
+
+def _moe(key, title, fmt, T, top_k, E, hidden, inter, seed):
+    lin = (Linear("gate_proj", inter, hidden, "x_moe"), Linear("up_proj", inter, hidden, "x_moe"),
+           Linear("down_proj", hidden, inter, "x_moe_down"))
+    acts = (("x_moe", hidden, "gauss"), ("x_moe_down", inter, "silu"))
+    return MoEWorkload(key, title, fmt, T, top_k, E, lin, acts, seed)
+
+
+MOE_WORKLOADS: Dict[str, MoEWorkload] = {
+    "moe_qwen": _moe("moe_qwen", "Qwen3-30B-A3B-shaped MoE experts (128 x {768x2048, 2048x768}) NVFP4, "
+                     "16x2048 tokens top-8", NVFP4, 32768, 8, 128, 2048, 768, 2001),
+    "moe_gptoss": _moe("moe_gptoss", "gpt-oss-120B-shaped MoE experts (128 x 2880x2880) MXFP4, 16x2048 tokens top-4",
+                       MXFP4, 32768, 4, 128, 2880, 2880, 2002),
+}
+
+
+def custom_moe(key: str, fmt: int, counts, N: int, K: int, seed: int, kind: str = "gauss") -> MoEWorkload:
+    """One expert linear [N, K] over len(counts) experts with fixed token counts."""
+    return MoEWorkload(key, f"{FMT_NAME[fmt]} {len(counts)} experts {N}x{K}", fmt, sum(counts), 1, len(counts),
+                       (Linear("w", N, K, "x"),), (("x", K, kind),), seed, counts=tuple(int(c) for c in counts))
+
+
+def gen_routing(wl: MoEWorkload) -> List[int]:
+    """Tokens routed to each expert (sums to wl.M): each of the T tokens picks top_k
+    distinct experts with probability proportional to the experts' popularity."""
+    if wl.counts is not None:
+        return list(wl.counts)
+    g = _gen(wl.seed, "router", "cpu")
+    pop = torch.exp(wl.route_sigma * torch.randn(wl.E, generator=g))
+    picks = torch.multinomial(pop.expand(wl.T, wl.E), wl.top_k, replacement=False, generator=g)
+    return torch.bincount(picks.reshape(-1), minlength=wl.E).tolist()
+
+
+def offsets_of(counts) -> List[int]:
+    out = [0]
+    for c in counts:
+        out.append(out[-1] + int(c))
+    return out
+
+
+@dataclasses.dataclass
+class Experts:
+    fmt: int
+    E: int
+    N: int
+    K: int
+    codes: torch.Tensor     # [E, N, K/2] uint8
+    scales: torch.Tensor    # [E, N, K/B] uint8
+    ws2: List[float]        # one tensor scale per expert
+
+
+def gen_experts(wl: MoEWorkload, lin: Linear, device="cpu") -> Experts:
+    """Every expert's weight drawn and RTN-quantized like gen_weight (one draw per expert)."""
+    codes = torch.empty(wl.E, lin.N, lin.K // 2, dtype=torch.uint8, device=device)
+    scales = torch.empty(wl.E, lin.N, lin.K // BLOCK[wl.fmt], dtype=torch.uint8, device=device)
+    ws2 = []
+    for e in range(wl.E):
+        g = _gen(wl.seed, f"W:{lin.name}:{e}", device)
+        w = torch.randn(lin.N, lin.K, generator=g, device=device, dtype=torch.float32) * wl.w_std
+        q = quantize_rtn(w, wl.fmt)
+        codes[e].copy_(q.codes)
+        scales[e].copy_(q.scales)
+        ws2.append(q.ws2)
+    return Experts(wl.fmt, wl.E, lin.N, lin.K, codes, scales, ws2)
