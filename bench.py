@@ -52,6 +52,9 @@ def parse_args():
                     help="skip the context legs (large-plane projection/merge ceiling, cuBLAS on pre-decoded weights)")
     ap.add_argument("--plane-only", action="store_true",
                     help="only the projection/merge ceiling on one 2^28-block plane (for profiling those kernels)")
+    ap.add_argument("--moe", default=None,
+                    help="time the grouped-expert step of an MoE workload instead (moe_qwen: Qwen3-30B-A3B-shaped "
+                         "NVFP4 experts; moe_gptoss: gpt-oss-120B-shaped MXFP4 experts)")
     ap.add_argument("--lowrank", action="store_true",
                     help="the paper's exact training step: the latent comes from the low-rank adapter "
                          "(sq_project_lowrank) and the adapter gradients follow the scale gradient "
@@ -653,6 +656,293 @@ def run_ours(args):
         print(json.dumps(line), flush=True)
 
 
+# --------------------------------------------------------------------- MoE experts
+
+class MoEState:
+    """Device-resident inputs and outputs of one grouped-expert step: every expert
+    linear (gate, up, down) of an MoE layer over the routed token rows."""
+
+    def __init__(self, wl, device):
+        import paper_2609_04526_gb300 as pkg
+        from paper_2609_04526_gb300 import synth
+        self.wl = wl
+        self.counts = synth.gen_routing(wl)
+        self.off = synth.offsets_of(self.counts)
+        M = self.off[-1]
+        self.acts = {name: synth.gen_act(wl, name, M=M, device=device) for name, _, _ in wl.acts}
+        self.lin = []
+        for lin in wl.linears:
+            ex = synth.gen_experts(wl, lin, device=device)
+            L = synth.gen_expert_latents(wl, lin, ex, device=device)
+            st = dict(lin=lin, ex=ex, latent=L, art=ex.scales.clone(), qbytes=torch.empty_like(ex.scales),
+                      mask=torch.empty_like(ex.scales), dY=synth.gen_dy(wl, lin, M=M, device=device),
+                      Y=torch.empty(M, lin.N, dtype=torch.bfloat16, device=device),
+                      dX=torch.empty(M, lin.K, dtype=torch.bfloat16, device=device),
+                      g=torch.empty(ex.scales.shape, dtype=torch.float32, device=device),
+                      nonfinite=torch.zeros(1, dtype=torch.int32, device=device),
+                      changed=torch.zeros(1, dtype=torch.int64, device=device))
+            # the forward and backward read the projected bytes; projection and merge read only ws2
+            st["gw"] = pkg.GroupedWeight(wl.fmt, wl.E, lin.N, lin.K, ex.codes, st["qbytes"], ex.ws2)
+            self.lin.append(st)
+
+    def inputs(self):
+        return {"acts": dict(self.acts), "dY": [st["dY"] for st in self.lin], "L": [st["latent"] for st in self.lin]}
+
+    def results(self):
+        out = []
+        for st in self.lin:
+            n = st["lin"].name
+            out += [("g:" + n, st["g"]), ("art:" + n, st["art"]), ("nf:" + n, st["nonfinite"]),
+                    ("ch:" + n, st["changed"])]
+        return out
+
+
+def run_moe_step(h, S, stream, events=None, ins=None):
+    """One grouped-expert step per linear: projection of every expert's latent plane,
+    forward, input gradient and masked scale gradient over all experts, merge."""
+    ins = S.inputs() if ins is None else ins
+    for i, st in enumerate(S.lin):
+        X, dY, L = ins["acts"][st["lin"].x], ins["dY"][i], ins["L"][i]
+        ev = events[i] if events is not None else None
+        gw = st["gw"]
+        calls = (lambda: h.sq_grouped_project_scales(gw, L, bytes_out=st["qbytes"], mask_out=st["mask"],
+                                                     nonfinite=st["nonfinite"], stream=stream),
+                 lambda: h.sq_grouped_fwd(gw, S.off, X, Y=st["Y"], stream=stream),
+                 lambda: h.sq_grouped_bwd_dx(gw, S.off, dY, dX=st["dX"], stream=stream),
+                 lambda: h.sq_grouped_scale_grad(gw, S.off, X, dY, mask=st["mask"], g=st["g"], stream=stream),
+                 lambda: h.sq_grouped_merge(gw, L, st["art"], changed=st["changed"], stream=stream))
+        for j, call in enumerate(calls):
+            if ev:
+                ev[j].record(stream)
+            call()
+        if ev:
+            ev[len(calls)].record(stream)
+
+
+def moe_context(h, S, stream, steps=3):
+    """Context legs of the MoE step: (1) the same contractions as a loop of dense
+    calls, one per expert (what a per-expert loop costs); (2) the dense kernels on
+    one weight over all routed rows at once (the same FLOPs without ragged experts:
+    the ceiling of the grouped launches)."""
+    wl = S.wl
+    off = S.off
+
+    def per_expert():
+        for st in S.lin:
+            X = S.acts[st["lin"].x]
+            for e in range(wl.E):
+                a, b = off[e], off[e + 1]
+                if b == a:
+                    continue
+                w = st["gw"].expert(e)
+                if w.scales.data_ptr() % 16:
+                    continue  # never for these workloads' planes (N * G is a multiple of 16)
+                h.sq_fwd(w, X[a:b], Y=st["Y"][a:b], stream=stream)
+                h.sq_bwd_dx(w, st["dY"][a:b], dX=st["dX"][a:b], stream=stream)
+                h.sq_scale_grad(w, X[a:b], st["dY"][a:b], mask=st["mask"][e], g=st["g"][e], stream=stream)
+
+    dense_w = [st["gw"].expert(0) for st in S.lin]
+
+    def dense_all_rows():
+        for st, w in zip(S.lin, dense_w):
+            X = S.acts[st["lin"].x]
+            h.sq_fwd(w, X, Y=st["Y"], stream=stream)
+            h.sq_bwd_dx(w, st["dY"], dX=st["dX"], stream=stream)
+            h.sq_scale_grad(w, X, st["dY"], mask=st["mask"][0], g=st["g"][0], stream=stream)
+
+    out = {}
+    for name, fn in (("per_expert_loop", per_expert), ("dense_same_rows", dense_all_rows)):
+        fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / steps
+        out[name] = {"value": wl.flops() / (ms / 1e3) / 1e12, "unit": UNIT, "ms_per_step": ms}
+    out["per_expert_loop"]["what"] = ("fwd, dX and scale gradient as one dense call per expert and linear "
+                                      f"({sum(1 for c in S.counts if c) * len(S.lin) * 3} launches per step)")
+    out["dense_same_rows"]["what"] = ("the dense kernels on one expert's weight over all routed rows at once: the same "
+                                      "FLOPs without per-expert raggedness (ceiling of the grouped launches)")
+    h.sq_sync(stream)
+    return out
+
+
+def moe_oracle_sample(S, n_experts=2, n_y=128, n_dx=128, n_rows=None, n_plane=1 << 14, seed=0):
+    """The float64 oracle on a bounded sample of the MoE step: a few experts of every
+    linear through oracle_sample's per-element rates, scaled to the whole step by
+    those experts' share of the step's FLOPs."""
+    import oracle
+    from paper_2609_04526_gb300 import synth
+    wl = S.wl
+    rng = np.random.default_rng(seed)
+    nz = [e for e in range(wl.E) if S.counts[e]]
+    experts = [int(e) for e in rng.choice(nz, min(n_experts, len(nz)), replace=False)]
+    n_rows = oracle.num_threads() if n_rows is None else n_rows
+    t_full = t_spent = 0.0
+    flops_sampled = 0
+    for st in S.lin:
+        lin = st["lin"]
+        X = S.acts[lin.x]
+        for e in experts:
+            a, b = S.off[e], S.off[e + 1]
+            sub = synth.custom(f"{wl.key}:{lin.name}:{e}", wl.fmt, b - a, lin.N, lin.K, seed=0)
+            sub_lin = sub.linears[0]
+            host = {sub_lin.name: dict(
+                codes=st["ex"].codes[e].cpu().numpy(), scales=st["ex"].scales[e].cpu().numpy(), ws2=st["ex"].ws2[e],
+                X=X[a:b].cpu().contiguous().view(torch.int16).numpy().view(np.uint16),
+                dY=st["dY"][a:b].cpu().contiguous().view(torch.int16).numpy().view(np.uint16),
+                mask=st["mask"][e].cpu().numpy(), latent=st["latent"][e].cpu().numpy())}
+            tf, ts, _ = oracle_sample(sub, host, [sub_lin], n_y=n_y, n_dx=n_dx, n_rows=n_rows, n_plane=n_plane,
+                                      seed=seed + e)
+            t_full += tf
+            t_spent += ts
+            flops_sampled += 6 * (b - a) * lin.N * lin.K
+    t_step = t_full * wl.flops() / flops_sampled
+    desc = (f"experts {experts} of every linear: {n_y} Y and {n_dx} dX elements, {n_rows} full scale-gradient rows "
+            f"and {n_plane} latents through projection and merge per expert linear; the step's time extrapolated "
+            "from per-element rates and those experts' share of the step's FLOPs")
+    return t_step, t_spent, desc
+
+
+def run_moe(args):
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import build, synth
+    world, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    build.build()
+    wl = synth.MOE_WORKLOADS[args.moe]
+    pk = peaks()
+    h = pkg.Handle()
+    stream = torch.cuda.current_stream()
+    S = MoEState(wl, "cuda")
+    kinds = KINDS
+    nl = len(S.lin)
+    for _ in range(args.warmup):
+        run_moe_step(h, S, stream)
+    h.sq_sync(stream)
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(len(kinds) + 1)] for _ in range(nl)]
+              for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    t_start.record(stream)
+    for k in range(args.steps):
+        run_moe_step(h, S, stream, events[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    h.sq_sync(stream)
+    ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
+    kind_ms = {k: 0.0 for k in kinds}
+    for k in range(args.steps):
+        for i in range(nl):
+            ev = events[k][i]
+            for j, kind in enumerate(kinds):
+                kind_ms[kind] += ev[j].elapsed_time(ev[j + 1])
+    M = S.off[-1]
+    fl = {k: sum(2 * M * st["lin"].N * st["lin"].K for st in S.lin) for k in ("fwd", "dx", "sgrad")}
+    blocks = sum(wl.E * st["lin"].N * (st["lin"].K // wl.block) for st in S.lin)
+    by = {"project": blocks * 6, "merge": blocks * 6}
+    kernels = {}
+    for kind in kinds:
+        t = kind_ms[kind] / args.steps / 1e3
+        if kind in fl:
+            ach = fl[kind] / t / 1e12
+            kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "TFLOP/s",
+                             "frac": ach / pk["bf16_sustained"]}
+        else:
+            ach = by[kind] / t / 1e9
+            kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
+    dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
+    value = wl.flops() * args.steps * world / (ms_total / 1e3) / 1e12
+
+    e2e = None
+    if not args.no_e2e:
+        sets = [S.inputs(), clone_input_set(S.inputs())]
+        host_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in flat_inputs(sets[0])]
+        for hst, dev in zip(host_in, flat_inputs(sets[0])):
+            hst.copy_(dev)
+        outs = [(t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for _, t in S.results()]
+        # + per linear: three expert tables (descriptors, tile starts, rows, ws2) of the grouped
+        # contractions and, for NVFP4, the experts' tensor scales for projection and merge
+        tables = nl * (3 * (268 * wl.E + 4) + (8 * wl.E if wl.fmt == 0 else 0))
+        h2d = sum(t.numel() * t.element_size() for t in host_in) + tables
+        d2h = sum(t.numel() * t.element_size() for t, _ in outs)
+        copy_stream = torch.cuda.Stream()
+        ready = [torch.cuda.Event(), torch.cuda.Event()]
+        free = [torch.cuda.Event(), torch.cuda.Event()]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+        def issue_copy(k):
+            b = k % 2
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(free[b] if k >= 2 else e0)
+                for hst, dev in zip(host_in, flat_inputs(sets[b])):
+                    dev.copy_(hst, non_blocking=True)
+                ready[b].record(copy_stream)
+
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        issue_copy(0)
+        for k in range(args.steps):
+            if k + 1 < args.steps:
+                issue_copy(k + 1)
+            stream.wait_event(ready[k % 2])
+            run_moe_step(h, S, stream, ins=sets[k % 2])
+            free[k % 2].record(stream)
+            for dev, hst in outs:
+                hst.copy_(dev, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        h.sq_sync(stream)
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+        e2e = {"value": wl.flops() * args.steps * world / (e2e_ms / 1e3) / 1e12, "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps,
+               "overlap": "inputs of step k+1 copied on a second stream while step k computes; the routing "
+                          "offsets and expert tables go host to device with every grouped call"}
+        del sets, host_in
+
+    context = {} if args.no_context else moe_context(h, S, stream)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.lib()
+        t_step, t_spent, desc = moe_oracle_sample(S)
+        cpu = {"value": wl.flops() / t_step / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+               "sample": desc, "sample_seconds": round(t_spent, 2), "extrapolated_step_seconds": round(t_step, 1)}
+    if rank == 0:
+        k = kernels[dom]
+        c = np.asarray(S.counts)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": f"{wl.key}: {wl.title}", "experts": wl.E, "top_k": wl.top_k, "tokens": wl.T,
+                       "routed_rows": int(M), "rows_per_expert": {"min": int(c.min()), "mean": float(c.mean()),
+                                                                  "max": int(c.max()), "empty": int((c == 0).sum())},
+                       "linears": {st["lin"].name: [st["lin"].N, st["lin"].K] for st in S.lin},
+                       "format": "nvfp4" if wl.fmt == 0 else "mxfp4",
+                       "l2": "inputs larger than L2 (routed activations + output gradients > 2 GB per step), no flush",
+                       "parallelism": f"replicas x{world}", "flops_per_step": wl.flops(),
+                       "step": "grouped experts: projection, fwd, dX, masked scale gradient, merge per linear"},
+            "roofline": {"bound": "tensor", "kernel": dom, "achieved": k["achieved"], "peak": pk["bf16_sustained"],
+                         "unit": "TFLOP/s", "frac": k["achieved"] / pk["bf16_sustained"], "traffic": None,
+                         "peak_source": f"{pk['source']} bf16 sustained"},
+            "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"],
+                                 "bf16_sustained": value / world / pk["bf16_sustained"]},
+            "kernels": kernels, "e2e": e2e, "cpu_baseline": cpu,
+            "gpu_launches": LAUNCHES_PER_LINEAR * nl * args.steps, "clocks": clk,
+        }
+        line.update(context)
+        print(json.dumps(line), flush=True)
+
+
 def run_reference(args):
     """The float64 CPU oracle, as it stands, on bounded samples of the same workload."""
     world, rank, local = dist_setup(args)
@@ -709,6 +999,8 @@ def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.moe:
+        run_moe(args)
     else:
         run_ours(args)
     if torch.distributed.is_available() and torch.distributed.is_initialized():

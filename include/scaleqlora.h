@@ -14,7 +14,8 @@
  *   sq_rollback        undo a merge with its on-grid delta (Sec. 5 Payoff 3)
  *   sq_swap_scales     scale-only hot-swap of the served adapter (Sec. 5)
  *   sq_count_diff      byte-level audit of two buffers (Sec. 5)
- *   sq_grouped_*       the three contractions over the experts of an MoE layer (Sec. 3)
+ *   sq_grouped_*       the contractions, projection and merge over the experts of an MoE
+ *                      linear, one launch each (Sec. 3)
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -266,6 +267,21 @@ sq_status sq_grouped_bwd_dx(sq_handle h, const sq_grouped_weight *w, const int64
  * g device fp32 [E, N, K/B]. The scale bytes are not read (scales may be NULL). */
 sq_status sq_grouped_scale_grad(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
                                 const uint16_t *dY, const uint8_t *mask, float *g, void *stream);
+
+/* Grid projection (sq_project_scales) of all E experts' latent planes in one
+ * launch: latent device fp32 [E, N, K/B], plane e projected with ws2[e];
+ * bytes_out device u8 [E, N, K/B]; mask_out device u8 [E, N, K/B] or NULL;
+ * nonfinite device int32 or NULL (the NaN count over all planes). codes and
+ * scales of w are not read (may be NULL). */
+sq_status sq_grouped_project_scales(sq_handle h, const sq_grouped_weight *w, const float *latent, uint8_t *bytes_out,
+                                    uint8_t *mask_out, int32_t *nonfinite, void *stream);
+
+/* Merge (sq_merge) of all E experts' latent planes in one launch into the scale
+ * planes scales_inout device u8 [E, N, K/B] (plane e with ws2[e]); ongrid_delta
+ * device fp32 [E, N, K/B] or NULL; changed_bytes device int64 or NULL (the count
+ * over all planes). No code byte is read or written. */
+sq_status sq_grouped_merge(sq_handle h, const sq_grouped_weight *w, const float *latent, uint8_t *scales_inout,
+                           float *ongrid_delta, int64_t *changed_bytes, void *stream);
 
 #ifdef __cplusplus
 }

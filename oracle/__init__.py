@@ -357,3 +357,28 @@ def grouped_scale_grad(fmt, codes, offsets, X_bits, dY_bits, mask=None, experts=
         if b > a:
             g[e] = scale_grad(fmt, codes[e], X_bits[a:b], dY_bits[a:b], None if mask is None else mask[e])
     return g
+
+
+def grouped_project(fmt, latent, ws2):
+    """(bytes, mask, nonfinite) of every expert's latent plane [E, N, G], plane e
+    projected with its own tensor scale ws2[e]."""
+    L = _c(latent, np.float32)
+    out = np.empty(L.shape, dtype=np.uint8)
+    mask = np.empty(L.shape, dtype=np.uint8)
+    nf = 0
+    for e in range(L.shape[0]):
+        out[e], mask[e], n = project(fmt, L[e], ws2[e])
+        nf += n
+    return out, mask, nf
+
+
+def grouped_merge(fmt, latent, scales, ws2):
+    """(new planes, on-grid deltas, changed bytes) of the merge of every expert's plane."""
+    L = _c(latent, np.float32)
+    new = np.empty(L.shape, dtype=np.uint8)
+    delta = np.empty(L.shape, dtype=np.float32)
+    ch = 0
+    for e in range(L.shape[0]):
+        new[e], delta[e], c = merge(fmt, L[e], scales[e], ws2[e])
+        ch += c
+    return new, delta, ch

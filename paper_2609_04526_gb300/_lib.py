@@ -28,7 +28,7 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
            "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
            "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
-           "sq_grouped_bwd_dx", "sq_grouped_scale_grad")
+           "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge")
 
 
 class SQError(RuntimeError):
@@ -83,6 +83,8 @@ def load() -> ctypes.CDLL:
     L.sq_grouped_fwd.argtypes = [vp, GW, OFF, vp, vp, vp]
     L.sq_grouped_bwd_dx.argtypes = [vp, GW, OFF, vp, vp, vp]
     L.sq_grouped_scale_grad.argtypes = [vp, GW, OFF, vp, vp, vp, vp, vp]
+    L.sq_grouped_project_scales.argtypes = [vp, GW, vp, vp, vp, vp, vp]
+    L.sq_grouped_merge.argtypes = [vp, GW, vp, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
@@ -314,3 +316,25 @@ class Handle:
         self._check(self._L.sq_grouped_scale_grad(self._h, ctypes.byref(wc), off, _ptr(X), _ptr(dY), _ptr(mask),
                                                   _ptr(g), _stream(stream)))
         return g
+
+    def sq_grouped_project_scales(self, w: GroupedWeight, latent: torch.Tensor, bytes_out: Optional[torch.Tensor] = None,
+                                  mask_out: Optional[torch.Tensor] = None, nonfinite: Optional[torch.Tensor] = None,
+                                  want_mask: bool = True, stream=None):
+        """Project every expert's latent plane [E, N, G] with its own ws2. Returns (bytes, mask)."""
+        if bytes_out is None:
+            bytes_out = torch.empty(latent.shape, dtype=torch.uint8, device=latent.device)
+        if mask_out is None and want_mask:
+            mask_out = torch.empty(latent.shape, dtype=torch.uint8, device=latent.device)
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_project_scales(self._h, ctypes.byref(wc), _ptr(latent), _ptr(bytes_out),
+                                                      _ptr(mask_out), _ptr(nonfinite), _stream(stream)))
+        return bytes_out, mask_out
+
+    def sq_grouped_merge(self, w: GroupedWeight, latent: torch.Tensor, scales_inout: torch.Tensor,
+                         ongrid_delta: Optional[torch.Tensor] = None, changed: Optional[torch.Tensor] = None,
+                         stream=None):
+        """Merge every expert's latent plane into scales_inout [E, N, G] with its own ws2."""
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_merge(self._h, ctypes.byref(wc), _ptr(latent), _ptr(scales_inout),
+                                             _ptr(ongrid_delta), _ptr(changed), _stream(stream)))
+        return scales_inout

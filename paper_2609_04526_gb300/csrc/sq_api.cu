@@ -129,6 +129,12 @@ sq_status make_act_map(sq_handle h, CUtensorMap *map, const void *ptr, int64_t i
                   CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
+// bf16 output [outer, inner] of the pair kernels, written by the epilogue warps as
+// 32-row x 32-column TMA store boxes (64-byte rows, 64-byte swizzle).
+sq_status make_out_map(sq_handle h, CUtensorMap *map, void *ptr, int64_t inner, int64_t outer) {
+  return make_map(h, map, ptr, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, inner, outer, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+}
+
 int block_of(int fmt) { return fmt == SQ_NVFP4 ? 16 : 32; }
 
 sq_status check_ws2(sq_handle h, int fmt, float ws2) {
@@ -190,17 +196,15 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
     // codes: 128 rows x 64 bytes (128 weights) per stage and CTA of the pair, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
-    // Y [M, N]: 32-row x 64-column store boxes (the epilogue's staging tiles), 128-byte swizzle
-    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->N, M, 64, 32,
-                    CU_TENSOR_MAP_SWIZZLE_128B));
+    // Y [M, N]: 32-row x 32-column store boxes (the epilogue's staging tiles), 64-byte swizzle
+    SQ_TRY(make_out_map(h, &tmOut, out, w->N, M));
   } else if (mode == sqi::MODE_DX) {
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));  // dY, 128 x 64 K-major boxes
     // codes: 128 contraction rows x 64 bytes (128 weights) per stage and CTA, 64-byte swizzle
     SQ_TRY(make_map(h, &tmB, w->codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, K2, w->N, 64, 128,
                     CU_TENSOR_MAP_SWIZZLE_64B));
-    // dX [M, K]: 32-row x 64-column store boxes, 128-byte swizzle
-    SQ_TRY(make_map(h, &tmOut, out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w->K, M, 64, 32,
-                    CU_TENSOR_MAP_SWIZZLE_128B));
+    // dX [M, K]: the same store boxes
+    SQ_TRY(make_out_map(h, &tmOut, out, w->K, M));
   } else {
     // dY and X as MN-major boxes of 64 features x kSgradBK tokens
     SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));
@@ -227,10 +231,9 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
 
 constexpr int kMaxExperts = 1 << 16;
 
-// Shape, scale and token-layout checks of a grouped call; on success `rows`
-// holds each expert's token count and M the total.
-sq_status check_grouped(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, bool need_scales,
-                        std::vector<int64_t> &rows, int64_t &M) {
+// Shape and tensor-scale checks of a grouped weight (codes and scales pointers
+// only where the call reads them).
+sq_status check_grouped_weight(sq_handle h, const sq_grouped_weight *w, bool need_codes, bool need_scales) {
   if (!w) return fail(h, SQ_ERR_INVALID_ARG, "grouped weight is NULL");
   if (w->E < 1 || w->E > kMaxExperts) return fail(h, SQ_ERR_INVALID_ARG, "E=%d must be in [1, 65536]", w->E);
   if (w->fmt != SQ_NVFP4 && w->fmt != SQ_MXFP4) return fail(h, SQ_ERR_INVALID_ARG, "unknown format %d", w->fmt);
@@ -248,9 +251,18 @@ sq_status check_grouped(sq_handle h, const sq_grouped_weight *w, const int64_t *
   // code rows of all experts are addressed with int32 TMA coordinates (plus one tile of overhang)
   if (static_cast<int64_t>(w->E) * w->N + 1024 > kMaxTokens)
     return fail(h, SQ_ERR_INVALID_ARG, "E * N = %lld code rows exceed 2^31 - 1024", (long long)w->E * w->N);
-  if (!w->codes || !aligned16(w->codes)) return fail(h, SQ_ERR_INVALID_ARG, "codes must be non-NULL and 16-byte aligned");
+  if (need_codes && (!w->codes || !aligned16(w->codes)))
+    return fail(h, SQ_ERR_INVALID_ARG, "codes must be non-NULL and 16-byte aligned");
   if (need_scales && (!w->scales || !aligned16(w->scales)))
     return fail(h, SQ_ERR_INVALID_ARG, "scales must be non-NULL and 16-byte aligned");
+  return SQ_OK;
+}
+
+// Weight and token-layout checks of a grouped contraction; on success `rows`
+// holds each expert's token count and M the total.
+sq_status check_grouped(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, bool need_scales,
+                        std::vector<int64_t> &rows, int64_t &M) {
+  SQ_TRY(check_grouped_weight(h, w, true, need_scales));
   if (!offsets) return fail(h, SQ_ERR_INVALID_ARG, "offsets is NULL");
   if (offsets[0] != 0) return fail(h, SQ_ERR_INVALID_ARG, "offsets[0] must be 0");
   rows.assign(w->E, 0);
@@ -291,14 +303,21 @@ sq_status acquire_table(sq_handle h, DeviceState *dev, size_t bytes, TableSlot *
 
 // One grouped contraction. FWD: a = X [M, K], out = Y [M, N]. DX: a = dY [M, N],
 // out = dX [M, K]. SGRAD: a = dY, b = X, out = g [E, N, G].
-sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const std::vector<int64_t> &rows,
-                      const int64_t *offsets, const uint16_t *a_ptr, const uint16_t *b_ptr, void *out,
-                      const uint8_t *mask, cudaStream_t stream) {
+// Grouped calls copy a host-built table on the stream: not while it is captured.
+sq_status check_not_capturing(sq_handle h, cudaStream_t stream) {
   cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
   cudaError_t e = cudaStreamIsCapturing(stream, &cap);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
   if (cap != cudaStreamCaptureStatusNone)
     return fail(h, SQ_ERR_UNSUPPORTED, "grouped calls copy a host-built expert table and cannot be graph-captured");
+  return SQ_OK;
+}
+
+sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const std::vector<int64_t> &rows,
+                      const int64_t *offsets, const uint16_t *a_ptr, const uint16_t *b_ptr, void *out,
+                      const uint8_t *mask, cudaStream_t stream) {
+  SQ_TRY(check_not_capturing(h, stream));
+  cudaError_t e;
   DeviceState *dev = nullptr;
   SQ_TRY(ensure_device(h, &dev));
   const int E = w->E;
@@ -335,12 +354,10 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
     const int64_t m = rows[x], r0 = offsets[x];
     if (mode == sqi::MODE_FWD) {
       SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * K, K, m, 64, sqi::kBM));
-      SQ_TRY(make_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * N, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                      N, m, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B));
+      SQ_TRY(make_out_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * N, N, m));
     } else if (mode == sqi::MODE_DX) {
       SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * N, N, m, 64, sqi::kBM));
-      SQ_TRY(make_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * K, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                      K, m, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B));
+      SQ_TRY(make_out_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * K, K, m));
     } else {
       SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * N, N, m, 64, sqi::kSgradBK));
       SQ_TRY(make_act_map(h, &maps[x].m[1], b_ptr + r0 * K, K, m, 64, sqi::kSgradBK));
@@ -379,6 +396,42 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
   cudaError_t e2 = cudaEventRecord(t->done, stream);
   if (e2 == cudaSuccess) t->pending = true;
   if (e != cudaSuccess) return cuda_fail(h, e, "grouped kernel launch");
+  if (e2 != cudaSuccess) return cuda_fail(h, e2, "cudaEventRecord(table)");
+  return SQ_OK;
+}
+
+// Projection (merge = false) or merge of the E experts' latent planes in one
+// launch. MXFP4 experts share ws2 = 1; NVFP4 experts' tensor scales go to the
+// device in an expert-table slot (one float per expert).
+sq_status run_grouped_plane(sq_handle h, const sq_grouped_weight *w, bool merge, const float *latent, uint8_t *bytes,
+                            uint8_t *mask_out, int32_t *nonfinite, float *delta, int64_t *changed,
+                            cudaStream_t stream) {
+  SQ_TRY(check_not_capturing(h, stream));
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const int64_t plane = static_cast<int64_t>(w->N) * (w->K / block_of(w->fmt));
+  const int64_t count = plane * w->E;
+  cudaError_t e;
+  if (w->fmt == SQ_MXFP4) {
+    e = merge ? sqi::launch_merge(w->fmt, count, 1.0f, latent, bytes, delta, changed, dev->sm_count, stream)
+              : sqi::launch_project(w->fmt, count, 1.0f, latent, bytes, mask_out, nonfinite, dev->sm_count, stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, merge ? "grouped merge launch" : "grouped projection launch");
+    return SQ_OK;
+  }
+  TableSlot *t = nullptr;
+  const size_t tbytes = static_cast<size_t>(w->E) * sizeof(float);
+  SQ_TRY(acquire_table(h, dev, tbytes, &t));
+  std::memcpy(t->host, w->ws2, tbytes);
+  if ((e = cudaMemcpyAsync(t->dev, t->host, tbytes, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+    return cuda_fail(h, e, "copying the expert tensor scales");
+  const float *ws2_dev = reinterpret_cast<const float *>(t->dev);
+  e = merge ? sqi::launch_merge(w->fmt, count, 1.0f, latent, bytes, delta, changed, dev->sm_count, stream, ws2_dev,
+                                plane)
+            : sqi::launch_project(w->fmt, count, 1.0f, latent, bytes, mask_out, nonfinite, dev->sm_count, stream,
+                                  ws2_dev, plane);
+  cudaError_t e2 = cudaEventRecord(t->done, stream);
+  if (e2 == cudaSuccess) t->pending = true;
+  if (e != cudaSuccess) return cuda_fail(h, e, merge ? "grouped merge launch" : "grouped projection launch");
   if (e2 != cudaSuccess) return cuda_fail(h, e2, "cudaEventRecord(table)");
   return SQ_OK;
 }
@@ -712,6 +765,36 @@ sq_status sq_grouped_bwd_dx(sq_handle h, const sq_grouped_weight *w, const int64
   SQ_TRY(check_buf(h, dY, "dY"));
   SQ_TRY(check_buf(h, dX, "dX"));
   return run_grouped(h, sqi::MODE_DX, w, rows, offsets, dY, nullptr, dX, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_project_scales(sq_handle h, const sq_grouped_weight *w, const float *latent, uint8_t *bytes_out,
+                                    uint8_t *mask_out, int32_t *nonfinite, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_grouped_weight(h, w, false, false));
+  SQ_TRY(check_buf(h, latent, "latent"));
+  SQ_TRY(check_buf(h, bytes_out, "bytes_out"));
+  if (mask_out && !aligned16(mask_out)) return fail(h, SQ_ERR_INVALID_ARG, "mask_out must be 16-byte aligned");
+  if (nonfinite && (reinterpret_cast<uintptr_t>(nonfinite) & 3u))
+    return fail(h, SQ_ERR_INVALID_ARG, "nonfinite must be 4-byte aligned");
+  return run_grouped_plane(h, w, false, latent, bytes_out, mask_out, nonfinite, nullptr, nullptr,
+                           static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_merge(sq_handle h, const sq_grouped_weight *w, const float *latent, uint8_t *scales_inout,
+                           float *ongrid_delta, int64_t *changed_bytes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_grouped_weight(h, w, false, false));
+  SQ_TRY(check_buf(h, latent, "latent"));
+  SQ_TRY(check_buf(h, scales_inout, "scales_inout"));
+  if (ongrid_delta && !aligned16(ongrid_delta)) return fail(h, SQ_ERR_INVALID_ARG, "ongrid_delta must be 16-byte aligned");
+  if (changed_bytes && (reinterpret_cast<uintptr_t>(changed_bytes) & 7u))
+    return fail(h, SQ_ERR_INVALID_ARG, "changed_bytes must be 8-byte aligned");
+  return run_grouped_plane(h, w, true, latent, scales_inout, nullptr, nullptr, ongrid_delta, changed_bytes,
+                           static_cast<cudaStream_t>(stream));
   SQ_GUARD_END
 }
 

@@ -562,13 +562,17 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
 //                   k-step loads two of them, one per 256-row half of the tile;
 //   decoded weights kStages slots of this CTA's 128 weight rows x one stage (32 KiB);
 //   packed codes    kCStages slots (8 KiB), released by the decode warps once read;
-//   output staging  one 4 KiB box per epilogue warp for the TMA stores of the result.
+//   output staging  one 2 KiB box (32 rows x 32 columns) per epilogue warp for the
+//                   TMA stores of the result.
 // A pair computes a 512 x 256 output tile: every decoded weight stage feeds the
 // MMAs of both 256-row halves, into two TMEM accumulators (all 512 columns), so
-// the decode-and-signal chain of a stage is covered by twice the tensor work.
+// the decode-and-signal chain of a stage is covered by twice the tensor work. The
+// next tile's MMAs wait for the epilogue to drain both accumulators; eight
+// epilogue warps (two per TMEM lane quadrant, one per column half) shorten that
+// wait.
 struct PairCfg {
-  static constexpr int kEpiWarps = 4;    // warps 0-3
-  static constexpr int kDecWarps = 16;   // warps 4-19: one 32-weight unit per thread per stage
+  static constexpr int kEpiWarps = 8;    // warps 0-7: warp w drains lane quadrant w % 4, column half w / 4
+  static constexpr int kDecWarps = 16;   // warps 8-23: one 32-weight unit per thread per stage
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;  // activation tiles
   static constexpr int kCodeWarp = kTmaWarp + 1;          // packed-code tiles
   static constexpr int kMmaWarp = kCodeWarp + 1;
@@ -583,8 +587,9 @@ struct PairCfg {
   static constexpr int kC = 128 * kBK / 2;  // 8 KiB: packed codes of that half (64-byte rows, 64-byte swizzle)
   static constexpr int kOffB = kAStages * kA;
   static constexpr int kOffC = kOffB + kStages * kB;
-  static constexpr int kOffS = kOffC + kCStages * kC;   // output staging: [kEpiWarps][32 x 64 bf16]
-  static constexpr int kOffBar = kOffS + kEpiWarps * 4096;
+  static constexpr int kOffS = kOffC + kCStages * kC;   // output staging: [kEpiWarps][32 x 32 bf16]
+  static constexpr int kBoxBytes = 32 * 32 * 2;
+  static constexpr int kOffBar = kOffS + kEpiWarps * kBoxBytes;
   static constexpr int kSmemBytes = kOffBar + 1024 + 1024;
   static constexpr uint32_t kATx = 2 * kA;                      // both CTAs' activation tiles, on the leader
   static constexpr uint32_t kSignalBytes = 4 * kDecWarps * 2;   // st.async bytes per stage: all decode warps, 2 CTAs
@@ -593,6 +598,7 @@ struct PairCfg {
 };
 static_assert(PairCfg::kSmemBytes <= 232448, "pair kernel exceeds the opt-in shared memory of one CTA");
 static_assert(PairCfg::kMTile == 2 * PairCfg::kTile, "a pair tile is two halves");
+static_assert(PairCfg::kEpiWarps == 8, "the epilogue maps warp w to lane quadrant w % 4 and column half w / 4");
 
 // Decode unit u (0..511) of this CTA's half at stage kb covers 32 consecutive
 // weights: row (u & 7) + 8 * (u >> 5) of the half, quarter (u >> 3) & 3 of its
@@ -923,19 +929,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       }
     }
   } else {
-    // ------------------------------------------------------ epilogue (warps 0-3, both CTAs)
+    // ------------------------------------------------------ epilogue (warps 0-7, both CTAs)
     // Drains accumulator 0 (rows 0-255 of the tile), releases it so the next
-    // tile's first MMAs can start, then drains accumulator 1. Each warp turns its
-    // 32 TMEM lanes x 64 columns into a bf16 box in shared memory (128-byte
-    // swizzle) and stores it with TMA, which writes whole 128-byte row segments
-    // and clips the ragged edges of the output.
-    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    // tile's first MMAs can start, then accumulator 1. Warp w reads TMEM lanes
+    // 32 (w % 4) .. +31 and columns 128 (w / 4) .. +127, 32 columns at a time:
+    // it scales and rounds them to bf16 into a 32 x 32 box in shared memory
+    // (64-byte swizzle) and stores the box with TMA, which writes whole row
+    // segments and clips the ragged edges of the output.
+    const int quad = warp & 3;
+    const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
+    const int cbase = (warp >> 2) * (C::kTile / 2);
     const int64_t Ng = MODE == MODE_FWD ? p.N : p.K;
     float scale = FMT == 0 ? p.ws2 : 1.0f;
     int64_t rows = p.M;
     const CUtensorMap *mO = &tmO;
-    const uint32_t box = smem_u32(smem + C::kOffS + warp * 4096);
-    const uint32_t row_base = box + lane * 128;  // this lane's 128-byte box row
+    const uint32_t box = smem_u32(smem + C::kOffS + warp * C::kBoxBytes);
+    const uint32_t row_base = box + lane * 64;  // this lane's 64-byte box row
     int tc = 0;
     int e = 0, e_seen = -1;
     for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
@@ -953,36 +962,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       for (int h = 0; h < 2 && ok; ++h) {
         if (!(ok = mbar_wait(&tfull[h], static_cast<uint32_t>(tc) & 1u, abort_flag, p.err))) break;
         tc_fence_after();
-        const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * warp;
+        const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * quad;
         const uint32_t t_buf = t_row + h * kTmemCols;
-        for (int c0 = 0; c0 < C::kTile; c0 += 64) {
 #pragma unroll 1
-          for (int half = 0; half < 2; ++half) {
-            uint32_t v[32];
-            tmem_ld32(t_buf + c0 + 32 * half, v);
-            tmem_ld_wait();
-            uint32_t packed[16];
+        for (int j = 0; j < C::kTile / 2; j += 32) {
+          const int c = cbase + j;
+          uint32_t v[32];
+          tmem_ld32(t_buf + c, v);
+          tmem_ld_wait();
+          uint32_t packed[16];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-              const __nv_bfloat162 h2 =
-                  __floats2bfloat162_rn(__uint_as_float(v[2 * e]) * scale, __uint_as_float(v[2 * e + 1]) * scale);
-              packed[e] = *reinterpret_cast<const uint32_t *>(&h2);
-            }
-            if (half == 0) {
-              if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
-              __syncwarp();
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const int chunk = 4 * half + q;
-              st_shared_v4(row_base + ((chunk ^ (lane & 7)) << 4), packed[4 * q], packed[4 * q + 1],
-                           packed[4 * q + 2], packed[4 * q + 3]);
-            }
+          for (int q = 0; q < 16; ++q) {
+            const __nv_bfloat162 h2 =
+                __floats2bfloat162_rn(__uint_as_float(v[2 * q]) * scale, __uint_as_float(v[2 * q + 1]) * scale);
+            packed[q] = *reinterpret_cast<const uint32_t *>(&h2);
           }
+          if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
+          __syncwarp();
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), packed[4 * q], packed[4 * q + 1],
+                         packed[4 * q + 2], packed[4 * q + 3]);
           fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
           __syncwarp();
           if (lane == 0) {
-            if (row < rows && col0 + c0 < Ng) tma_store_2d(mO, box, col0 + c0, row);
+            if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
             bulk_commit_group();
           }
         }

@@ -75,15 +75,20 @@ cudaError_t launch_grouped(const GroupedArgs &a, const CUtensorMap &tmCodes, int
 // Launch one contraction. tmA is the TMA descriptor of the streamed bf16
 // activations; tmB that of the packed codes (MODE_FWD / MODE_DX) or of the second
 // bf16 operand (MODE_SGRAD); tmOut that of the bf16 output (MODE_FWD / MODE_DX:
-// 32-row x 64-column boxes, 128-byte swizzle; null for MODE_SGRAD).
+// 32-row x 32-column boxes, 64-byte swizzle; null for MODE_SGRAD).
 cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap *tmOut,
                         int sm_count, cudaStream_t stream);
 
+// Projection / merge of `count` latents. With ws2_per (device, one float per
+// expert) the latents are the planes of several experts, `plane` (a multiple of
+// 16) elements each, and element i uses ws2_per[i / plane] instead of ws2.
 cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *latent, uint8_t *bytes_out,
-                           uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream);
+                           uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream,
+                           const float *ws2_per = nullptr, int64_t plane = 0);
 
 cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *scales_inout,
-                         float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream);
+                         float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream,
+                         const float *ws2_per = nullptr, int64_t plane = 0);
 
 // Rollback of a merge by its on-grid delta (in place, counting changed bytes), and
 // copy a -> b (write) or only count the bytes in which a and b differ.

@@ -116,8 +116,18 @@ __device__ __forceinline__ void warp_add_i64(int64_t *counter, uint32_t v) {
     atomicAdd(reinterpret_cast<unsigned long long *>(counter), static_cast<unsigned long long>(v));
 }
 
+// Planes of several experts in one launch (ws2_per non-null): element i belongs
+// to expert i / plane and takes that expert's tensor scale; plane is a multiple
+// of 16, so one 16-element vector never straddles two experts.
+__device__ __forceinline__ void expert_scale(const float *ws2_per, int64_t plane, int64_t i, float &ws2, float &cap) {
+  if (!ws2_per) return;
+  ws2 = __ldg(ws2_per + i / plane);
+  cap = 448.0f * ws2;  // the same IEEE fp32 product as the host's single-plane cap
+}
+
 template <int FMT>
-__global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, float ws2, float cap,
+__global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, float ws2_all, float cap_all,
+                                                              const float *__restrict__ ws2_per, int64_t plane,
                                                               const float *__restrict__ latent,
                                                               uint8_t *__restrict__ bytes_out,
                                                               uint8_t *__restrict__ mask_out,
@@ -126,6 +136,8 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   uint32_t nan_count = 0;
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    float ws2 = ws2_all, cap = cap_all;
+    expert_scale(ws2_per, plane, 16 * v, ws2, cap);
     const float4 *src = reinterpret_cast<const float4 *>(latent) + 4 * v;
     float L[16];
 #pragma unroll
@@ -151,6 +163,8 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
   // ragged tail (< 16 values) by the first threads of block 0
   if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
     const int64_t i = nvec * 16 + threadIdx.x;
+    float ws2 = ws2_all, cap = cap_all;
+    expert_scale(ws2_per, plane, i, ws2, cap);
     uint32_t b, m, n;
     project_one<FMT>(latent[i], ws2, cap, b, m, n);
     bytes_out[i] = static_cast<uint8_t>(b);
@@ -161,7 +175,8 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
 }
 
 template <int FMT>
-__global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float ws2, float cap,
+__global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float ws2_all, float cap_all,
+                                                            const float *__restrict__ ws2_per, int64_t plane,
                                                             const float *__restrict__ latent,
                                                             uint8_t *__restrict__ scales,
                                                             float *__restrict__ delta,
@@ -170,6 +185,8 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   uint32_t n_changed = 0;
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    float ws2 = ws2_all, cap = cap_all;
+    expert_scale(ws2_per, plane, 16 * v, ws2, cap);
     const float4 *src = reinterpret_cast<const float4 *>(latent) + 4 * v;
     float L[16];
 #pragma unroll
@@ -202,6 +219,8 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   }
   if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
     const int64_t i = nvec * 16 + threadIdx.x;
+    float ws2 = ws2_all, cap = cap_all;
+    expert_scale(ws2_per, plane, i, ws2, cap);
     uint32_t b, m, n;
     project_one<FMT>(latent[i], ws2, cap, b, m, n);
     const uint32_t o = scales[i];
@@ -525,7 +544,8 @@ unsigned grid_for(int64_t count, int sm_count) {
 }  // namespace
 
 cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *latent, uint8_t *bytes_out,
-                           uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream) {
+                           uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream,
+                           const float *ws2_per, int64_t plane) {
   if (nonfinite) {
     cudaError_t e = cudaMemsetAsync(nonfinite, 0, sizeof(int32_t), stream);
     if (e != cudaSuccess) return e;
@@ -534,14 +554,17 @@ cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *laten
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
   const unsigned grid = grid_for(count, sm_count);
   if (fmt == 0)
-    sq_project_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, latent, bytes_out, mask_out, nonfinite);
+    sq_project_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, bytes_out, mask_out,
+                                                        nonfinite);
   else
-    sq_project_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, latent, bytes_out, mask_out, nonfinite);
+    sq_project_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, bytes_out, mask_out,
+                                                        nonfinite);
   return cudaGetLastError();
 }
 
 cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent, uint8_t *scales_inout,
-                         float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream) {
+                         float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream,
+                         const float *ws2_per, int64_t plane) {
   if (changed) {
     cudaError_t e = cudaMemsetAsync(changed, 0, sizeof(int64_t), stream);
     if (e != cudaSuccess) return e;
@@ -550,9 +573,11 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
   const unsigned grid = grid_for(count, sm_count);
   if (fmt == 0)
-    sq_merge_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, latent, scales_inout, ongrid_delta, changed);
+    sq_merge_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, scales_inout,
+                                                      ongrid_delta, changed);
   else
-    sq_merge_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, latent, scales_inout, ongrid_delta, changed);
+    sq_merge_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, scales_inout,
+                                                      ongrid_delta, changed);
   return cudaGetLastError();
 }
 

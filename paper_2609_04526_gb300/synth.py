@@ -270,6 +270,9 @@ class MoEWorkload:
     counts: Optional[tuple] = None  # fixed per-expert token counts (tests); else drawn by the router
     w_std: float = 0.02
     dy_std: float = 1e-3
+    latent_rel_rms: float = 0.021   # as Workload
+    latent_rank: int = 54           # the paper's MoE scale rank (scale r54)
+    above_ceiling_frac: float = 1e-3
 
     @property
     def block(self) -> int:
@@ -348,3 +351,13 @@ def gen_experts(wl: MoEWorkload, lin: Linear, device="cpu") -> Experts:
         scales[e].copy_(q.scales)
         ws2.append(q.ws2)
     return Experts(wl.fmt, wl.E, lin.N, lin.K, codes, scales, ws2)
+
+
+def gen_expert_latents(wl: MoEWorkload, lin: Linear, ex: Experts, device="cpu") -> torch.Tensor:
+    """Latent effective scales [E, N, G] of every expert (gen_latent per expert, each
+    with its own draw)."""
+    out = torch.empty(ex.scales.shape, dtype=torch.float32, device=device)
+    for e in range(ex.E):
+        w = Weight(ex.fmt, ex.N, ex.K, ex.codes[e], ex.scales[e], ex.ws2[e])
+        out[e].copy_(gen_latent(wl, dataclasses.replace(lin, name=f"{lin.name}:{e}"), w, device=device))
+    return out

@@ -222,3 +222,37 @@ def test_grouped_invalid_args_and_capture(h):
             h.sq_grouped_fwd(gw, [0, 4, 8], X, Y=Y, stream=s)
     assert ei.value.status == -2
     h.sq_sync()
+
+
+@pytest.mark.parametrize("key,fmt,E,N,K", [("p_nv", NV, 5, 40, 96 * 2), ("p_mx", MX, 3, 24, 96),
+                                           ("p_nv_qwen_gate", NV, 128, 768, 2048)])
+def test_grouped_projection_and_merge_bit_exact(h, key, fmt, E, N, K):
+    """Every expert's plane projected / merged with its own ws2 in one launch: bytes,
+    masks, deltas and counters bit-exact against the oracle (NaN and above-ceiling
+    latents included)."""
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom_moe(key, fmt, [1] * E, N, K, seed=E + N)
+    lin = wl.linears[0]
+    ex = synth.gen_experts(wl, lin, device="cuda")
+    gw = pkg.GroupedWeight(ex.fmt, ex.E, ex.N, ex.K, None, None, ex.ws2)
+    L = synth.gen_expert_latents(wl, lin, ex, device="cuda")
+    L[0, 0, 0] = float("nan")
+    L[E - 1, N - 1, 1] = float("inf")
+    nf = torch.zeros(1, dtype=torch.int32, device="cuda")
+    b, m = h.sq_grouped_project_scales(gw, L, nonfinite=nf)
+    art = ex.scales.clone()
+    delta = torch.empty_like(L)
+    ch = torch.zeros(1, dtype=torch.int64, device="cuda")
+    h.sq_grouped_merge(gw, L, art, ongrid_delta=delta, changed=ch)
+    h.sq_sync()
+    Lh = host(L)
+    rb, rm, rnf = oracle.grouped_project(fmt, Lh, ex.ws2)
+    assert np.array_equal(host(b), rb) and np.array_equal(host(m), rm) and int(nf.item()) == rnf
+    rnew, rdelta, rch = oracle.grouped_merge(fmt, Lh, host(ex.scales), ex.ws2)
+    assert np.array_equal(host(art), rnew) and int(ch.item()) == rch
+    dh = host(delta)
+    assert np.array_equal(np.isnan(dh), np.isnan(rdelta))
+    ok = ~np.isnan(rdelta)
+    assert np.array_equal(dh[ok].view(np.uint32), rdelta[ok].view(np.uint32))
+    assert (rb != host(ex.scales)).mean() > 0.005                      # the latents moved bytes

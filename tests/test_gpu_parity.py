@@ -26,7 +26,7 @@ def h():
 
 
 SMALL = [
-    # key, fmt, M, N, K      (pair tiles: 512 x 256 with 128-deep k-steps; scale-gradient tiles: 128 x 256)
+    # key, fmt, M, N, K      (pair tiles: 512 x 256 with 128-deep k-steps; scale-gradient tiles: 256 x 256)
     ("c1", NV, 64, 256, 512),
     ("nv_ragged", NV, 300, 392, 608),
     ("mx_ragged", MX, 257, 264, 544),
@@ -35,6 +35,8 @@ SMALL = [
     ("mx_tall", MX, 1000, 520, 96),
     ("nv_long_k", NV, 70, 136, 2080),
     ("nv_long_m", NV, 1500, 40, 256),
+    ("nv_last_tile_short", NV, 600, 264, 320),    # last 512-row tile: 88 rows
+    ("mx_last_tile_one_half", MX, 1280, 136, 256),  # last 512-row tile: exactly 256 rows
 ]
 
 

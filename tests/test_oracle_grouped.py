@@ -159,3 +159,26 @@ def test_no_tokens_at_all(oracle_mod):
     assert oracle_mod.grouped_fwd(MX, codes, scales, ws2, off, Xb).shape == (0, 8)
     g = oracle_mod.grouped_scale_grad(MX, codes, off, Xb, dYb)
     assert g.shape == (3, 8, 2) and not g.any()
+
+
+def test_grouped_projection_uses_each_experts_tensor_scale(oracle_mod):
+    """Inside the E4M3 range the projected byte of plane e is torch's RNE float8
+    cast of fl32(L / ws2[e]); latents placed on the grid of one expert's ws2 land
+    on different bytes under another's, so a plane projected with the wrong
+    expert's scale fails. The merge then rewrites exactly the bytes that differ."""
+    rng = np.random.default_rng(65)
+    E, N, G = 3, 16, 8
+    ws2 = [2.0 ** -7, 3.0 * 2.0 ** -9, 2.0 ** -5]
+    L = np.empty((E, N, G), dtype=np.float32)
+    for e in range(E):
+        L[e] = (rng.uniform(0.02, 400.0, size=(N, G)) * ws2[e]).astype(np.float32)
+    b, m, nf = oracle_mod.grouped_project(NV, L, ws2)
+    for e in range(E):
+        q = (L[e] / np.float32(ws2[e])).astype(np.float32)
+        ref = torch.from_numpy(q).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+        assert np.array_equal(b[e], ref) and (m[e] == 1).all()
+    assert nf == 0
+    assert not np.array_equal(oracle_mod.grouped_project(NV, L, ws2[::-1])[0], b)
+    old = rng.integers(0x30, 0x70, size=(E, N, G), dtype=np.uint8)
+    new, delta, ch = oracle_mod.grouped_merge(NV, L, old, ws2)
+    assert np.array_equal(new, b) and ch == int((old != b).sum())
