@@ -80,8 +80,8 @@ cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
                         int sm_count, cudaStream_t stream);
 
 // Projection / merge of `count` latents. With ws2_per (device, one float per
-// expert) the latents are the planes of several experts, `plane` (a multiple of
-// 16) elements each, and element i uses ws2_per[i / plane] instead of ws2.
+// expert; NVFP4 only) the latents are the planes of several experts, `plane` (a
+// multiple of 16) elements each, and element i uses ws2_per[i / plane] instead of ws2.
 cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *latent, uint8_t *bytes_out,
                            uint8_t *mask_out, int32_t *nonfinite, int sm_count, cudaStream_t stream,
                            const float *ws2_per = nullptr, int64_t plane = 0);

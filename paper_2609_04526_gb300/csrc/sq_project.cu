@@ -116,16 +116,15 @@ __device__ __forceinline__ void warp_add_i64(int64_t *counter, uint32_t v) {
     atomicAdd(reinterpret_cast<unsigned long long *>(counter), static_cast<unsigned long long>(v));
 }
 
-// Planes of several experts in one launch (ws2_per non-null): element i belongs
+// Planes of several experts in one launch (PER instantiations): element i belongs
 // to expert i / plane and takes that expert's tensor scale; plane is a multiple
 // of 16, so one 16-element vector never straddles two experts.
 __device__ __forceinline__ void expert_scale(const float *ws2_per, int64_t plane, int64_t i, float &ws2, float &cap) {
-  if (!ws2_per) return;
   ws2 = __ldg(ws2_per + i / plane);
   cap = 448.0f * ws2;  // the same IEEE fp32 product as the host's single-plane cap
 }
 
-template <int FMT>
+template <int FMT, bool PER>
 __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, float ws2_all, float cap_all,
                                                               const float *__restrict__ ws2_per, int64_t plane,
                                                               const float *__restrict__ latent,
@@ -137,7 +136,7 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
   uint32_t nan_count = 0;
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
     float ws2 = ws2_all, cap = cap_all;
-    expert_scale(ws2_per, plane, 16 * v, ws2, cap);
+    if (PER) expert_scale(ws2_per, plane, 16 * v, ws2, cap);
     const float4 *src = reinterpret_cast<const float4 *>(latent) + 4 * v;
     float L[16];
 #pragma unroll
@@ -164,7 +163,7 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
   if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
     const int64_t i = nvec * 16 + threadIdx.x;
     float ws2 = ws2_all, cap = cap_all;
-    expert_scale(ws2_per, plane, i, ws2, cap);
+    if (PER) expert_scale(ws2_per, plane, i, ws2, cap);
     uint32_t b, m, n;
     project_one<FMT>(latent[i], ws2, cap, b, m, n);
     bytes_out[i] = static_cast<uint8_t>(b);
@@ -174,7 +173,7 @@ __global__ void __launch_bounds__(kThreads) sq_project_kernel(int64_t count, flo
   if (nonfinite) warp_add_i32(nonfinite, nan_count);
 }
 
-template <int FMT>
+template <int FMT, bool PER>
 __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float ws2_all, float cap_all,
                                                             const float *__restrict__ ws2_per, int64_t plane,
                                                             const float *__restrict__ latent,
@@ -186,7 +185,7 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   uint32_t n_changed = 0;
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
     float ws2 = ws2_all, cap = cap_all;
-    expert_scale(ws2_per, plane, 16 * v, ws2, cap);
+    if (PER) expert_scale(ws2_per, plane, 16 * v, ws2, cap);
     const float4 *src = reinterpret_cast<const float4 *>(latent) + 4 * v;
     float L[16];
 #pragma unroll
@@ -220,7 +219,7 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
     const int64_t i = nvec * 16 + threadIdx.x;
     float ws2 = ws2_all, cap = cap_all;
-    expert_scale(ws2_per, plane, i, ws2, cap);
+    if (PER) expert_scale(ws2_per, plane, i, ws2, cap);
     uint32_t b, m, n;
     project_one<FMT>(latent[i], ws2, cap, b, m, n);
     const uint32_t o = scales[i];
@@ -553,12 +552,15 @@ cudaError_t launch_project(int fmt, int64_t count, float ws2, const float *laten
   if (count == 0) return cudaSuccess;
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
   const unsigned grid = grid_for(count, sm_count);
-  if (fmt == 0)
-    sq_project_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, bytes_out, mask_out,
-                                                        nonfinite);
+  if (ws2_per)  // several NVFP4 experts, each with its own tensor scale
+    sq_project_kernel<0, true><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, bytes_out,
+                                                              mask_out, nonfinite);
+  else if (fmt == 0)
+    sq_project_kernel<0, false><<<grid, kThreads, 0, stream>>>(count, ws2, cap, nullptr, 0, latent, bytes_out,
+                                                               mask_out, nonfinite);
   else
-    sq_project_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, bytes_out, mask_out,
-                                                        nonfinite);
+    sq_project_kernel<1, false><<<grid, kThreads, 0, stream>>>(count, ws2, cap, nullptr, 0, latent, bytes_out,
+                                                               mask_out, nonfinite);
   return cudaGetLastError();
 }
 
@@ -572,12 +574,15 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
   if (count == 0) return cudaSuccess;
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
   const unsigned grid = grid_for(count, sm_count);
-  if (fmt == 0)
-    sq_merge_kernel<0><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, scales_inout,
-                                                      ongrid_delta, changed);
+  if (ws2_per)  // several NVFP4 experts, each with its own tensor scale
+    sq_merge_kernel<0, true><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, scales_inout,
+                                                            ongrid_delta, changed);
+  else if (fmt == 0)
+    sq_merge_kernel<0, false><<<grid, kThreads, 0, stream>>>(count, ws2, cap, nullptr, 0, latent, scales_inout,
+                                                             ongrid_delta, changed);
   else
-    sq_merge_kernel<1><<<grid, kThreads, 0, stream>>>(count, ws2, cap, ws2_per, plane, latent, scales_inout,
-                                                      ongrid_delta, changed);
+    sq_merge_kernel<1, false><<<grid, kThreads, 0, stream>>>(count, ws2, cap, nullptr, 0, latent, scales_inout,
+                                                             ongrid_delta, changed);
   return cudaGetLastError();
 }
 
