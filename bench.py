@@ -662,10 +662,11 @@ class MoEState:
     """Device-resident inputs and outputs of one grouped-expert step: every expert
     linear (gate, up, down) of an MoE layer over the routed token rows."""
 
-    def __init__(self, wl, device):
+    def __init__(self, wl, device, lowrank=False):
         import paper_2609_04526_gb300 as pkg
         from paper_2609_04526_gb300 import synth
         self.wl = wl
+        self.lowrank = lowrank
         self.counts = synth.gen_routing(wl)
         self.off = synth.offsets_of(self.counts)
         M = self.off[-1]
@@ -683,6 +684,11 @@ class MoEState:
                       changed=torch.zeros(1, dtype=torch.int64, device=device))
             # the forward and backward read the projected bytes; projection and merge read only ws2
             st["gw"] = pkg.GroupedWeight(wl.fmt, wl.E, lin.N, lin.K, ex.codes, st["qbytes"], ex.ws2)
+            if lowrank:  # every expert's adapter over its frozen base plane (rank 54, the paper's MoE rank)
+                st["gw_base"] = pkg.GroupedWeight(wl.fmt, wl.E, lin.N, lin.K, None, ex.scales, ex.ws2)
+                st["B"], st["A"], st["aor"] = synth.gen_expert_adapters(wl, lin, ex, device=device)
+                st["dB"] = torch.empty(st["B"].shape, dtype=torch.float32, device=device)
+                st["dA"] = torch.empty(st["A"].shape, dtype=torch.float32, device=device)
             self.lin.append(st)
 
     def inputs(self):
@@ -705,12 +711,21 @@ def run_moe_step(h, S, stream, events=None, ins=None):
         X, dY, L = ins["acts"][st["lin"].x], ins["dY"][i], ins["L"][i]
         ev = events[i] if events is not None else None
         gw = st["gw"]
-        calls = (lambda: h.sq_grouped_project_scales(gw, L, bytes_out=st["qbytes"], mask_out=st["mask"],
-                                                     nonfinite=st["nonfinite"], stream=stream),
+        if S.lowrank:
+            project = lambda: h.sq_grouped_project_lowrank(st["gw_base"], st["B"], st["A"], st["aor"],
+                                                           bytes_out=st["qbytes"], mask_out=st["mask"],
+                                                           nonfinite=st["nonfinite"], latent_out=L, stream=stream)
+        else:
+            project = lambda: h.sq_grouped_project_scales(gw, L, bytes_out=st["qbytes"], mask_out=st["mask"],
+                                                          nonfinite=st["nonfinite"], stream=stream)
+        calls = [project,
                  lambda: h.sq_grouped_fwd(gw, S.off, X, Y=st["Y"], stream=stream),
                  lambda: h.sq_grouped_bwd_dx(gw, S.off, dY, dX=st["dX"], stream=stream),
-                 lambda: h.sq_grouped_scale_grad(gw, S.off, X, dY, mask=st["mask"], g=st["g"], stream=stream),
-                 lambda: h.sq_grouped_merge(gw, L, st["art"], changed=st["changed"], stream=stream))
+                 lambda: h.sq_grouped_scale_grad(gw, S.off, X, dY, mask=st["mask"], g=st["g"], stream=stream)]
+        if S.lowrank:
+            calls.append(lambda: h.sq_grouped_lowrank_grad(st["g"], st["B"], st["A"], st["aor"], dB=st["dB"],
+                                                           dA=st["dA"], stream=stream))
+        calls.append(lambda: h.sq_grouped_merge(gw, L, st["art"], changed=st["changed"], stream=stream))
         for j, call in enumerate(calls):
             if ev:
                 ev[j].record(stream)
@@ -817,8 +832,11 @@ def run_moe(args):
     pk = peaks()
     h = pkg.Handle()
     stream = torch.cuda.current_stream()
-    S = MoEState(wl, "cuda")
-    kinds = KINDS
+    if args.lowrank:
+        args.no_e2e = True
+        args.no_cpu_baseline = True
+    S = MoEState(wl, "cuda", lowrank=args.lowrank)
+    kinds = KINDS_LOWRANK if args.lowrank else KINDS
     nl = len(S.lin)
     for _ in range(args.warmup):
         run_moe_step(h, S, stream)
@@ -848,6 +866,10 @@ def run_moe(args):
     fl = {k: sum(2 * M * st["lin"].N * st["lin"].K for st in S.lin) for k in ("fwd", "dx", "sgrad")}
     blocks = sum(wl.E * st["lin"].N * (st["lin"].K // wl.block) for st in S.lin)
     by = {"project": blocks * 6, "merge": blocks * 6}
+    if args.lowrank:  # as kernel_work: base byte in, byte + mask + latent out, the factors; g in, dB and dA out
+        factors = sum(wl.E * (st["lin"].N + st["lin"].K // wl.block) * st["B"].shape[2] * 2 for st in S.lin)
+        by["project"] = blocks * 7 + factors
+        by["adapter_grad"] = blocks * 4 + factors * 3
     kernels = {}
     for kind in kinds:
         t = kind_ms[kind] / args.steps / 1e3
@@ -930,14 +952,17 @@ def run_moe(args):
                        "format": "nvfp4" if wl.fmt == 0 else "mxfp4",
                        "l2": "inputs larger than L2 (routed activations + output gradients > 2 GB per step), no flush",
                        "parallelism": f"replicas x{world}", "flops_per_step": wl.flops(),
-                       "step": "grouped experts: projection, fwd, dX, masked scale gradient, merge per linear"},
+                       "step": ("grouped experts: rank-54 adapters of all experts, projection, fwd, dX, masked scale "
+                                "gradient, adapter gradients, merge per linear" if args.lowrank else
+                                "grouped experts: projection, fwd, dX, masked scale gradient, merge per linear")},
             "roofline": {"bound": "tensor", "kernel": dom, "achieved": k["achieved"], "peak": pk["bf16_sustained"],
                          "unit": "TFLOP/s", "frac": k["achieved"] / pk["bf16_sustained"], "traffic": None,
                          "peak_source": f"{pk['source']} bf16 sustained"},
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"],
                                  "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels, "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": LAUNCHES_PER_LINEAR * nl * args.steps, "clocks": clk,
+            "gpu_launches": (LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl * args.steps,
+            "clocks": clk,
         }
         line.update(context)
         print(json.dumps(line), flush=True)

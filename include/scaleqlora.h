@@ -268,6 +268,26 @@ sq_status sq_grouped_bwd_dx(sq_handle h, const sq_grouped_weight *w, const int64
 sq_status sq_grouped_scale_grad(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
                                 const uint16_t *dY, const uint8_t *mask, float *g, void *stream);
 
+/* The low-rank adapters of all E experts in one launch (Sec. 3 "MoE: a batched
+ * grouped-expert kernel": one batched product forms every expert's Delta S):
+ * expert e's latent eff' = eff + (alpha/r) B[e] A[e], formed and projected
+ * exactly as sq_project_lowrank with ws2[e]. w->scales are the frozen base planes
+ * [E, N, K/B] (read only; codes are not read); B device bf16 [E, N, r]; A device
+ * bf16 [E, r, K/B]; bytes_out, mask_out (or NULL), latent_out (fp32, or NULL)
+ * device [E, N, K/B]; nonfinite device int32 or NULL (count over all experts).
+ * Requires E <= 65535, 1 <= r <= 256 and finite alpha_over_r. */
+sq_status sq_grouped_project_lowrank(sq_handle h, const sq_grouped_weight *w, int32_t r, float alpha_over_r,
+                                     const uint16_t *B, const uint16_t *A, uint8_t *bytes_out, uint8_t *mask_out,
+                                     int32_t *nonfinite, float *latent_out, void *stream);
+
+/* sq_lowrank_grad for E experts in one set of launches: g device fp32 [E, N, G];
+ * B [E, N, r], A [E, r, G] bf16; dB device fp32 [E, N, r] or NULL; dA device fp32
+ * [E, r, G] or NULL (not both NULL). Same arithmetic, order and empty-sum rules
+ * per expert; 1 <= E <= 65535. Uses the handle's scratch, like sq_lowrank_grad. */
+sq_status sq_grouped_lowrank_grad(sq_handle h, int32_t E, int64_t N, int64_t G, int32_t r, float alpha_over_r,
+                                  const float *g, const uint16_t *B, const uint16_t *A, float *dB, float *dA,
+                                  void *stream);
+
 /* Grid projection (sq_project_scales) of all E experts' latent planes in one
  * launch: latent device fp32 [E, N, K/B], plane e projected with ws2[e];
  * bytes_out device u8 [E, N, K/B]; mask_out device u8 [E, N, K/B] or NULL;

@@ -382,3 +382,29 @@ def grouped_merge(fmt, latent, scales, ws2):
         new[e], delta[e], c = merge(fmt, L[e], scales[e], ws2[e])
         ch += c
     return new, delta, ch
+
+
+def grouped_project_lowrank(fmt, base_scales, B_bits, A_bits, ws2, alpha_over_r):
+    """Every expert's adapter latent and projection (project_lowrank per expert):
+    base [E, N, G] u8, B [E, N, r] and A [E, r, G] bf16 bits, ws2 one value per expert.
+    Returns (bytes, mask, nonfinite, latent) over all experts."""
+    base = _c(base_scales, np.uint8)
+    E = base.shape[0]
+    out = np.empty(base.shape, dtype=np.uint8)
+    mask = np.empty(base.shape, dtype=np.uint8)
+    latent = np.empty(base.shape, dtype=np.float32)
+    nf = 0
+    for e in range(E):
+        out[e], mask[e], n, latent[e] = project_lowrank(fmt, base[e], B_bits[e], A_bits[e], ws2[e], alpha_over_r)
+        nf += n
+    return out, mask, nf, latent
+
+
+def grouped_lowrank_grad(gm, B_bits, A_bits, alpha_over_r):
+    """Every expert's adapter gradients (lowrank_grad per expert): gm [E, N, G]."""
+    E = gm.shape[0]
+    dB = np.empty((E,) + B_bits.shape[1:], dtype=np.float64)
+    dA = np.empty((E,) + A_bits.shape[1:], dtype=np.float64)
+    for e in range(E):
+        dB[e], dA[e] = lowrank_grad(gm[e], B_bits[e], A_bits[e], alpha_over_r)
+    return dB, dA

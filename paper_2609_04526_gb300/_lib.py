@@ -28,7 +28,8 @@ STATUS = {0: "SQ_OK", -1: "SQ_ERR_INVALID_ARG", -2: "SQ_ERR_UNSUPPORTED", -3: "S
 EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_sync", "sq_fwd", "sq_bwd_dx",
            "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
            "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
-           "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge")
+           "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
+           "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad")
 
 
 class SQError(RuntimeError):
@@ -85,6 +86,8 @@ def load() -> ctypes.CDLL:
     L.sq_grouped_scale_grad.argtypes = [vp, GW, OFF, vp, vp, vp, vp, vp]
     L.sq_grouped_project_scales.argtypes = [vp, GW, vp, vp, vp, vp, vp]
     L.sq_grouped_merge.argtypes = [vp, GW, vp, vp, vp, vp, vp]
+    L.sq_grouped_project_lowrank.argtypes = [vp, GW, i32, f32, vp, vp, vp, vp, vp, vp, vp]
+    L.sq_grouped_lowrank_grad.argtypes = [vp, i32, i64, i64, i32, f32, vp, vp, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
@@ -338,3 +341,32 @@ class Handle:
         self._check(self._L.sq_grouped_merge(self._h, ctypes.byref(wc), _ptr(latent), _ptr(scales_inout),
                                              _ptr(ongrid_delta), _ptr(changed), _stream(stream)))
         return scales_inout
+
+    def sq_grouped_project_lowrank(self, w: GroupedWeight, B: torch.Tensor, A: torch.Tensor, alpha_over_r: float,
+                                   bytes_out: Optional[torch.Tensor] = None, mask_out: Optional[torch.Tensor] = None,
+                                   nonfinite: Optional[torch.Tensor] = None, latent_out: Optional[torch.Tensor] = None,
+                                   stream=None):
+        """Every expert's adapter latent eff + (alpha/r) B[e] A[e] over its base plane w.scales[e],
+        projected with its ws2. B [E, N, r], A [E, r, G] bf16. Returns (bytes, mask, latent)."""
+        r = B.shape[2]
+        if bytes_out is None:
+            bytes_out = torch.empty(w.scales.shape, dtype=torch.uint8, device=w.scales.device)
+        wc, keep = w._c()
+        self._check(self._L.sq_grouped_project_lowrank(self._h, ctypes.byref(wc), r, alpha_over_r, _ptr(B), _ptr(A),
+                                                       _ptr(bytes_out), _ptr(mask_out), _ptr(nonfinite),
+                                                       _ptr(latent_out), _stream(stream)))
+        return bytes_out, mask_out, latent_out
+
+    def sq_grouped_lowrank_grad(self, g: torch.Tensor, B: torch.Tensor, A: torch.Tensor, alpha_over_r: float,
+                                dB: Optional[torch.Tensor] = None, dA: Optional[torch.Tensor] = None,
+                                want_dB: bool = True, want_dA: bool = True, stream=None):
+        """Adapter gradients of every expert: g [E, N, G] fp32 -> dB [E, N, r], dA [E, r, G]."""
+        E, N, G = g.shape
+        r = B.shape[2]
+        if dB is None and want_dB:
+            dB = torch.empty(E, N, r, dtype=torch.float32, device=g.device)
+        if dA is None and want_dA:
+            dA = torch.empty(E, r, G, dtype=torch.float32, device=g.device)
+        self._check(self._L.sq_grouped_lowrank_grad(self._h, E, N, G, r, alpha_over_r, _ptr(g), _ptr(B), _ptr(A),
+                                                    _ptr(dB), _ptr(dA), _stream(stream)))
+        return dB, dA

@@ -230,6 +230,7 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
 // ------------------------------------------------------------------ grouped (experts)
 
 constexpr int kMaxExperts = 1 << 16;
+constexpr int kMaxGridZ = 65535;  // experts of the adapter launches (grid z)
 
 // Shape and tensor-scale checks of a grouped weight (codes and scales pointers
 // only where the call reads them).
@@ -795,6 +796,87 @@ sq_status sq_grouped_merge(sq_handle h, const sq_grouped_weight *w, const float 
     return fail(h, SQ_ERR_INVALID_ARG, "changed_bytes must be 8-byte aligned");
   return run_grouped_plane(h, w, true, latent, scales_inout, nullptr, nullptr, ongrid_delta, changed_bytes,
                            static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_project_lowrank(sq_handle h, const sq_grouped_weight *w, int32_t r, float alpha_over_r,
+                                     const uint16_t *B, const uint16_t *A, uint8_t *bytes_out, uint8_t *mask_out,
+                                     int32_t *nonfinite, float *latent_out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_grouped_weight(h, w, false, true));
+  if (w->E > kMaxGridZ) return fail(h, SQ_ERR_INVALID_ARG, "E=%d exceeds 65535 for the adapter launches", w->E);
+  if (r < 1 || r > sqi::kMaxLowRank) return fail(h, SQ_ERR_INVALID_ARG, "rank r=%d must be in [1, 256]", r);
+  if (!std::isfinite(alpha_over_r)) return fail(h, SQ_ERR_INVALID_ARG, "alpha_over_r must be finite");
+  SQ_TRY(check_buf(h, B, "B"));
+  SQ_TRY(check_buf(h, A, "A"));
+  SQ_TRY(check_buf(h, bytes_out, "bytes_out"));
+  if (mask_out && !aligned16(mask_out)) return fail(h, SQ_ERR_INVALID_ARG, "mask_out must be 16-byte aligned");
+  if (latent_out && !aligned16(latent_out)) return fail(h, SQ_ERR_INVALID_ARG, "latent_out must be 16-byte aligned");
+  if (nonfinite && (reinterpret_cast<uintptr_t>(nonfinite) & 3u))
+    return fail(h, SQ_ERR_INVALID_ARG, "nonfinite must be 4-byte aligned");
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SQ_TRY(check_not_capturing(h, st));
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const int64_t N = w->N, G = w->K / block_of(w->fmt);
+  cudaError_t e;
+  if (w->fmt == SQ_MXFP4) {
+    e = sqi::launch_project_lowrank(w->fmt, N, G, r, 1.0f, alpha_over_r, w->scales, B, A, bytes_out, mask_out,
+                                    nonfinite, latent_out, st, w->E, nullptr);
+    if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter projection launch");
+    return SQ_OK;
+  }
+  TableSlot *t = nullptr;
+  const size_t tbytes = static_cast<size_t>(w->E) * sizeof(float);
+  SQ_TRY(acquire_table(h, dev, tbytes, &t));
+  std::memcpy(t->host, w->ws2, tbytes);
+  if ((e = cudaMemcpyAsync(t->dev, t->host, tbytes, cudaMemcpyHostToDevice, st)) != cudaSuccess)
+    return cuda_fail(h, e, "copying the expert tensor scales");
+  e = sqi::launch_project_lowrank(w->fmt, N, G, r, 1.0f, alpha_over_r, w->scales, B, A, bytes_out, mask_out,
+                                  nonfinite, latent_out, st, w->E, reinterpret_cast<const float *>(t->dev));
+  cudaError_t e2 = cudaEventRecord(t->done, st);
+  if (e2 == cudaSuccess) t->pending = true;
+  if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter projection launch");
+  if (e2 != cudaSuccess) return cuda_fail(h, e2, "cudaEventRecord(table)");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_grouped_lowrank_grad(sq_handle h, int32_t E, int64_t N, int64_t G, int32_t r, float alpha_over_r,
+                                  const float *g, const uint16_t *B, const uint16_t *A, float *dB, float *dA,
+                                  void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (E < 1 || E > kMaxGridZ) return fail(h, SQ_ERR_INVALID_ARG, "E=%d must be in [1, 65535]", E);
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  if (r < 1 || r > sqi::kMaxLowRank) return fail(h, SQ_ERR_INVALID_ARG, "rank r=%d must be in [1, 256]", r);
+  if (!std::isfinite(alpha_over_r)) return fail(h, SQ_ERR_INVALID_ARG, "alpha_over_r must be finite");
+  if (!dB && !dA) return fail(h, SQ_ERR_INVALID_ARG, "dB and dA are both NULL");
+  if (dB && N > 0 && !aligned16(dB)) return fail(h, SQ_ERR_INVALID_ARG, "dB must be non-NULL and 16-byte aligned");
+  if (dA && G > 0 && !aligned16(dA)) return fail(h, SQ_ERR_INVALID_ARG, "dA must be non-NULL and 16-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (N == 0 || G == 0) {  // empty sums: the gradients are zero
+    if (dB && N > 0 &&
+        (e = cudaMemsetAsync(dB, 0, static_cast<size_t>(E) * N * r * sizeof(float), st)) != cudaSuccess)
+      return cuda_fail(h, e, "cudaMemsetAsync");
+    if (dA && G > 0 &&
+        (e = cudaMemsetAsync(dA, 0, static_cast<size_t>(E) * G * r * sizeof(float), st)) != cudaSuccess)
+      return cuda_fail(h, e, "cudaMemsetAsync");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, g, "g"));
+  SQ_TRY(check_buf(h, B, "B"));
+  SQ_TRY(check_buf(h, A, "A"));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count, E)));
+  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
+                               dev->sm_count, st, E);
+  if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter gradient launch");
+  return SQ_OK;
   SQ_GUARD_END
 }
 

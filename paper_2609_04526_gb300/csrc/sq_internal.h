@@ -99,14 +99,17 @@ cudaError_t launch_swap_or_diff(int64_t count, const uint8_t *a, uint8_t *b, boo
 
 // Low-rank scale adapter (Sec. 3 "Scale-QLoRA forward"): latent eff + (alpha/r) B A
 // projected onto the grid; and the gradients of B and A from the masked scale
-// gradient, through `workspace` (lowrank_grad_workspace bytes).
+// gradient, through `workspace` (lowrank_grad_workspace bytes). With experts > 1
+// the planes and factors of that many experts follow each other in memory (one
+// launch for all); ws2_per (device, NVFP4) gives each expert's tensor scale.
 cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float ws2, float alpha_over_r,
                                    const uint8_t *base, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
-                                   uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream);
-size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count);
+                                   uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream,
+                                   int experts = 1, const float *ws2_per = nullptr);
+size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count, int experts = 1);
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
-                                cudaStream_t stream);
+                                cudaStream_t stream, int experts = 1);
 constexpr int kMaxLowRank = 256;  // r limit of the adapter kernels
 
 // Device-side error codes written to the error word.

@@ -336,6 +336,10 @@ __global__ void __launch_bounds__(kThreads) sq_swap_or_diff_kernel(int64_t count
 // B [N, r] and A [r, G] bf16, formed in fp32 in a fixed order -- eff = fl32(decoded
 // base byte * ws2) (scale_value), acc = fused multiply-adds over j = 0 .. r-1 from 0,
 // eff' = fma(alpha/r, acc, eff) -- and projected exactly as sq_project_kernel.
+// The adapters of the E experts of an MoE linear (Sec. 3 "MoE: a batched
+// grouped-expert kernel") run in the same launches: expert e's planes and factors
+// follow expert e - 1's, and grid z (with the contraction chunk for the products)
+// selects the expert; a dense call is the case E = 1.
 // The three adapter kernels are register-tiled fp32 CUDA-core products: a CTA of 256
 // threads owns a 64 x 64 output tile, its operands staged in shared memory as fp32,
 // and each thread accumulates a 4 x 4 sub-tile (rows ty*4 .. +3, columns tx + 16c),
@@ -347,14 +351,27 @@ __device__ __forceinline__ float bf16_bits(uint16_t h) { return __uint_as_float(
 
 template <int FMT>
 __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
-    int64_t N, int64_t G, int r, float ws2, float cap, float aor, const uint8_t *__restrict__ base,
-    const uint16_t *__restrict__ B, const uint16_t *__restrict__ A, uint8_t *__restrict__ bytes_out,
-    uint8_t *__restrict__ mask_out, int32_t *__restrict__ nonfinite, float *__restrict__ latent_out) {
+    int64_t N, int64_t G, int r, float ws2, float cap, const float *__restrict__ ws2_per, float aor,
+    const uint8_t *__restrict__ base, const uint16_t *__restrict__ B, const uint16_t *__restrict__ A,
+    uint8_t *__restrict__ bytes_out, uint8_t *__restrict__ mask_out, int32_t *__restrict__ nonfinite,
+    float *__restrict__ latent_out) {
   extern __shared__ float lr_smem[];
   float *sB = lr_smem;            // [kT rows][r]
   float *sA = lr_smem + kT * r;   // [r][kT columns]
   const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kT;
   const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kT;
+  // expert blockIdx.z: its planes, factors and (NVFP4 experts) tensor scale
+  const int64_t e = blockIdx.z, plane = N * G;
+  base += e * plane;
+  B += e * N * r;
+  A += e * r * G;
+  bytes_out += e * plane;
+  if (mask_out) mask_out += e * plane;
+  if (latent_out) latent_out += e * plane;
+  if (ws2_per) {
+    ws2 = __ldg(ws2_per + e);
+    cap = 448.0f * ws2;  // the same IEEE fp32 product as the host's single-plane cap
+  }
   for (int i = threadIdx.x; i < kT * r; i += kThreads) {
     const int64_t n = n0 + i / r;
     sB[i] = n < N ? bf16_bits(B[n * r + i % r]) : 0.f;
@@ -412,37 +429,46 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
 constexpr int kKStep = 16;  // contraction indices per staged step
 
 // Operand element (row i of the output, contraction index k) for the two products.
+// `estride` is the distance between two experts' operands; expert(e) is expert e's.
 struct DbLeft {  // g[n = i][b = k]
   const float *g;
-  int64_t G;
+  int64_t G, estride;
   __device__ float operator()(int64_t i, int64_t k) const { return g[i * G + k]; }
+  __device__ DbLeft expert(int64_t e) const { return DbLeft{g + e * estride, G, estride}; }
 };
 struct DbRight {  // A[j = i][b = k]
   const uint16_t *A;
-  int64_t G;
+  int64_t G, estride;
   __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(A[i * G + k]); }
+  __device__ DbRight expert(int64_t e) const { return DbRight{A + e * estride, G, estride}; }
 };
 struct DaLeft {  // B[n = k][j = i]
   const uint16_t *B;
-  int r;
+  int64_t r, estride;
   __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(B[k * r + i]); }
+  __device__ DaLeft expert(int64_t e) const { return DaLeft{B + e * estride, r, estride}; }
 };
 struct DaRight {  // g[n = k][b = i]
   const float *g;
-  int64_t G;
+  int64_t G, estride;
   __device__ float operator()(int64_t i, int64_t k) const { return g[k * G + i]; }
+  __device__ DaRight expert(int64_t e) const { return DaRight{g + e * estride, G, estride}; }
 };
 
-// partial[z][i][j] = sum_{k in chunk z} L(i, k) R(j, k), i < rows, j < cols.
+// partial[e][c][i][j] = sum_{k in chunk c} L_e(i, k) R_e(j, k), i < rows, j < cols,
+// for expert e = blockIdx.z / chunks and chunk c = blockIdx.z % chunks.
 template <class LeftT, class RightT, bool LEFT_K_FAST, bool RIGHT_K_FAST>
 __global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t rows, int64_t cols, int64_t kdim,
-                                                                      int64_t kchunk, LeftT left, RightT right,
-                                                                      float *__restrict__ partial) {
+                                                                      int64_t kchunk, int64_t chunks, LeftT left_all,
+                                                                      RightT right_all, float *__restrict__ partial) {
   __shared__ float sl[2][kKStep][kT + 1];  // [buffer][k][i]
   __shared__ float sr[2][kKStep][kT + 1];  // [buffer][k][j]
+  const int64_t expert = blockIdx.z / chunks, chunk = blockIdx.z % chunks;
+  const LeftT left = left_all.expert(expert);
+  const RightT right = right_all.expert(expert);
   const int64_t i0 = static_cast<int64_t>(blockIdx.x) * kT;
   const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kT;
-  const int64_t kb = static_cast<int64_t>(blockIdx.z) * kchunk;
+  const int64_t kb = chunk * kchunk;
   const int64_t ke = kdim < kb + kchunk ? kdim : kb + kchunk;
   const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
   // staging map: 4 elements of each operand per thread and step; consecutive threads
@@ -510,15 +536,19 @@ __global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t ro
     }
 }
 
-// out[i] = scale * sum over chunks z (in order) of partial[z][i].
-__global__ void __launch_bounds__(kThreads) sq_adapter_reduce_kernel(int64_t count, int64_t chunks, float scale,
-                                                                     const float *__restrict__ partial,
+// out[e][i] = scale * sum over chunks c (in order) of partial[e][c][i], for the
+// `experts` outputs of `count` elements each.
+__global__ void __launch_bounds__(kThreads) sq_adapter_reduce_kernel(int64_t count, int64_t experts, int64_t chunks,
+                                                                     float scale, const float *__restrict__ partial,
                                                                      float *__restrict__ out) {
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < count;
-       i += static_cast<int64_t>(gridDim.x) * kThreads) {
+  const int64_t total = count * experts;
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; t < total;
+       t += static_cast<int64_t>(gridDim.x) * kThreads) {
+    const int64_t e = t / count, i = t - e * count;
+    const float *src = partial + e * chunks * count + i;
     float s = 0.f;
-    for (int64_t c = 0; c < chunks; ++c) s += partial[c * count + i];
-    out[i] = scale * s;
+    for (int64_t c = 0; c < chunks; ++c) s += src[c * count];
+    out[t] = scale * s;
   }
 }
 
@@ -588,68 +618,76 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
 
 cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float ws2, float alpha_over_r,
                                    const uint8_t *base, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
-                                   uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream) {
+                                   uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream,
+                                   int experts, const float *ws2_per) {
   if (nonfinite) {
     cudaError_t e = cudaMemsetAsync(nonfinite, 0, sizeof(int32_t), stream);
     if (e != cudaSuccess) return e;
   }
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
-  const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT));
+  const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT),
+                  static_cast<unsigned>(experts));
   const size_t smem = static_cast<size_t>(2 * kT) * r * sizeof(float);  // <= 128 KiB for r <= 256
   cudaError_t e;
   if (fmt == 0) {
     if ((e = cudaFuncSetAttribute(sq_project_lowrank_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess)
       return e;
-    sq_project_lowrank_kernel<0><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
-                                                                   bytes_out, mask_out, nonfinite, latent_out);
+    sq_project_lowrank_kernel<0><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, ws2_per, alpha_over_r, base,
+                                                                   B, A, bytes_out, mask_out, nonfinite, latent_out);
   } else {
     if ((e = cudaFuncSetAttribute(sq_project_lowrank_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess)
       return e;
-    sq_project_lowrank_kernel<1><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, alpha_over_r, base, B, A,
-                                                                   bytes_out, mask_out, nonfinite, latent_out);
+    sq_project_lowrank_kernel<1><<<grid, kThreads, smem, stream>>>(N, G, r, ws2, cap, nullptr, alpha_over_r, base,
+                                                                   B, A, bytes_out, mask_out, nonfinite, latent_out);
   }
   return cudaGetLastError();
 }
 
-// Workspace of the adapter gradients: the partial products of dB and of dA.
-size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count) {
-  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT), ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT);
+// Workspace of the adapter gradients: the partial products of dB and of dA (all experts).
+size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count, int experts) {
+  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT) * experts;
+  const int64_t ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT) * experts;
   const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);
-  return static_cast<size_t>(cb * N * r + ca * r * G) * sizeof(float);
+  return static_cast<size_t>(experts) * static_cast<size_t>(cb * N * r + ca * r * G) * sizeof(float);
 }
 
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
-                                cudaStream_t stream) {
-  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT), ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT);
+                                cudaStream_t stream, int experts) {
+  const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT) * experts;
+  const int64_t ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT) * experts;
   const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);
-  float *pb = workspace, *pa = workspace + cb * N * r;
+  float *pb = workspace, *pa = workspace + static_cast<int64_t>(experts) * cb * N * r;
   const unsigned reduce_cap = static_cast<unsigned>(sm_count) * kCtasPerSm;
   cudaError_t e;
   if (dB) {  // rows n, columns j, contraction b: g is b-contiguous, A is b-contiguous
     const int64_t kc = ((G + cb - 1) / cb + kKStep - 1) / kKStep * kKStep;
+    const int64_t chunks = (G + kc - 1) / kc;
     const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((r + kT - 1) / kT),
-                    static_cast<unsigned>((G + kc - 1) / kc));
+                    static_cast<unsigned>(chunks * experts));
     sq_adapter_product_kernel<DbLeft, DbRight, true, true><<<grid, kThreads, 0, stream>>>(
-        N, r, G, kc, DbLeft{g, G}, DbRight{A, G}, pb);
+        N, r, G, kc, chunks, DbLeft{g, G, N * G}, DbRight{A, G, static_cast<int64_t>(r) * G}, pb);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int64_t count = N * r;
-    const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((count + kThreads - 1) / kThreads, reduce_cap));
-    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, grid.z, alpha_over_r, pb, dB);
+    const unsigned blocks =
+        static_cast<unsigned>(std::min<int64_t>((count * experts + kThreads - 1) / kThreads, reduce_cap));
+    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, experts, chunks, alpha_over_r, pb, dB);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (dA) {  // rows j, columns b, contraction n: B is j-contiguous (row index fast), g is b-contiguous
     const int64_t kc = ((N + ca - 1) / ca + kKStep - 1) / kKStep * kKStep;
+    const int64_t chunks = (N + kc - 1) / kc;
     const dim3 grid(static_cast<unsigned>((r + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT),
-                    static_cast<unsigned>((N + kc - 1) / kc));
+                    static_cast<unsigned>(chunks * experts));
     sq_adapter_product_kernel<DaLeft, DaRight, false, false><<<grid, kThreads, 0, stream>>>(
-        r, G, N, kc, DaLeft{B, r}, DaRight{g, G}, pa);
+        r, G, N, kc, chunks, DaLeft{B, r, N * r}, DaRight{g, G, N * G}, pa);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int64_t count = static_cast<int64_t>(r) * G;
-    const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((count + kThreads - 1) / kThreads, reduce_cap));
-    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, grid.z, alpha_over_r, pa, dA);
+    const unsigned blocks =
+        static_cast<unsigned>(std::min<int64_t>((count * experts + kThreads - 1) / kThreads, reduce_cap));
+    sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, experts, chunks, alpha_over_r, pa, dA);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -361,3 +361,21 @@ def gen_expert_latents(wl: MoEWorkload, lin: Linear, ex: Experts, device="cpu") 
         w = Weight(ex.fmt, ex.N, ex.K, ex.codes[e], ex.scales[e], ex.ws2[e])
         out[e].copy_(gen_latent(wl, dataclasses.replace(lin, name=f"{lin.name}:{e}"), w, device=device))
     return out
+
+
+def gen_expert_adapters(wl: MoEWorkload, lin: Linear, ex: Experts, r: Optional[int] = None, alpha: float = 16.0,
+                        device="cpu"):
+    """Low-rank adapter factors of every expert (gen_adapter per expert, each with its
+    own draw): B [E, N, r] and A [E, r, G] bf16 and the shared alpha/r."""
+    r = wl.latent_rank if r is None else r
+    G = ex.K // BLOCK[ex.fmt]
+    B = torch.empty(ex.E, ex.N, r, dtype=torch.bfloat16, device=device)
+    A = torch.empty(ex.E, r, G, dtype=torch.bfloat16, device=device)
+    aor = alpha / r
+    for e in range(ex.E):
+        w = Weight(ex.fmt, ex.N, ex.K, ex.codes[e], ex.scales[e], ex.ws2[e])
+        Be, Ae, aor = gen_adapter(wl, dataclasses.replace(lin, name=f"{lin.name}:{e}"), w, r=r, alpha=alpha,
+                                  device=device)
+        B[e].copy_(Be)
+        A[e].copy_(Ae)
+    return B, A, aor

@@ -256,3 +256,48 @@ def test_grouped_projection_and_merge_bit_exact(h, key, fmt, E, N, K):
     ok = ~np.isnan(rdelta)
     assert np.array_equal(dh[ok].view(np.uint32), rdelta[ok].view(np.uint32))
     assert (rb != host(ex.scales)).mean() > 0.005                      # the latents moved bytes
+
+
+@pytest.mark.parametrize("key,fmt,E,N,K,r", [("a_nv", NV, 5, 40, 192, 13), ("a_mx", MX, 3, 24, 96 * 4, 7),
+                                             ("a_qwen_gate", NV, 128, 768, 2048, 54)])
+def test_grouped_adapter_projection_bit_exact_and_gradients(h, key, fmt, E, N, K, r):
+    """Every expert's adapter latent, byte, mask and NaN count bit-exact against the
+    oracle in one launch; the adapter gradients of all experts within the bar and
+    the same on a second run."""
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom_moe(key, fmt, [1] * E, N, K, seed=E * 7 + r)
+    lin = wl.linears[0]
+    ex = synth.gen_experts(wl, lin, device="cuda")
+    gw = pkg.GroupedWeight(ex.fmt, ex.E, ex.N, ex.K, None, ex.scales, ex.ws2)
+    B, A, aor = synth.gen_expert_adapters(wl, lin, ex, r=r, device="cuda")
+    B_clean = B.clone()
+    if fmt == NV:
+        B[1, 0, 0] = float("nan")                                      # one NaN latent row in expert 1
+    G = K // (16 if fmt == NV else 32)
+    mask = torch.empty(E, N, G, dtype=torch.uint8, device="cuda")
+    latent = torch.empty(E, N, G, dtype=torch.float32, device="cuda")
+    nf = torch.zeros(1, dtype=torch.int32, device="cuda")
+    b, _, _ = h.sq_grouped_project_lowrank(gw, B, A, aor, mask_out=mask, nonfinite=nf, latent_out=latent)
+    gen = torch.Generator(device="cuda").manual_seed(E + N)
+    g = torch.randn(E, N, G, device="cuda", generator=gen) * mask.float()
+    B = B_clean                                                         # finite factors for the gradients
+    dB, dA = h.sq_grouped_lowrank_grad(g, B, A, aor)
+    dB2, dA2 = h.sq_grouped_lowrank_grad(g, B, A, aor)
+    h.sq_sync()
+    Bn = B_clean.clone()
+    if fmt == NV:
+        Bn[1, 0, 0] = float("nan")
+    rb, rm, rnf, rL = oracle.grouped_project_lowrank(fmt, host(ex.scales), hbits(Bn), hbits(A), ex.ws2, aor)
+    gL = host(latent)
+    nan = np.isnan(rL)
+    assert np.array_equal(np.isnan(gL), nan)
+    assert np.array_equal(gL[~nan].view(np.uint32), rL[~nan].view(np.uint32)), "latent differs from the oracle"
+    assert np.array_equal(host(b), rb) and np.array_equal(host(mask), rm) and int(nf.item()) == rnf
+    if fmt == NV:  # a 2% relative move crosses E4M3 grid midpoints, never the E8M0 ones (factor sqrt 2)
+        assert (rb != host(ex.scales)).mean() > 0.005
+    gh = host(g)
+    rdB, rdA = oracle.grouped_lowrank_grad(gh, hbits(B), hbits(A), aor)
+    assert_close(host(dB), rdB, what="dB")
+    assert_close(host(dA), rdA, what="dA")
+    assert torch.equal(dB, dB2) and torch.equal(dA, dA2), "adapter gradients are not reproducible"

@@ -182,3 +182,33 @@ def test_grouped_projection_uses_each_experts_tensor_scale(oracle_mod):
     old = rng.integers(0x30, 0x70, size=(E, N, G), dtype=np.uint8)
     new, delta, ch = oracle_mod.grouped_merge(NV, L, old, ws2)
     assert np.array_equal(new, b) and ch == int((old != b).sum())
+
+
+def test_grouped_adapter_uses_each_experts_factors_and_scale(oracle_mod):
+    """An expert with B = 0 keeps its base plane byte for byte while the others move;
+    relabelling the experts (base plane, factors, ws2 together) relabels every
+    output; the gradients of expert e depend only on expert e's g, B and A."""
+    rng = np.random.default_rng(66)
+    E, N, G, r, aor = 4, 16, 24, 5, 0.5
+    base = rng.integers(0x30, 0x68, size=(E, N, G), dtype=np.uint8)
+    ws2 = [2.0 ** -7, 2.0 ** -6, 3.0 * 2.0 ** -9, 2.0 ** -8]
+    Bf = rng.normal(0, 1, (E, N, r)) * 0.05 * np.array(ws2)[:, None, None] * 40
+    Bf[2] = 0.0
+    Bb = torch.from_numpy(Bf.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    Ab = torch.from_numpy(rng.normal(0, 1, (E, r, G)).astype(np.float32)).to(torch.bfloat16).view(
+        torch.int16).numpy().view(np.uint16)
+    b, m, nf, L = oracle_mod.grouped_project_lowrank(NV, base, Bb, Ab, ws2, aor)
+    assert np.array_equal(b[2], base[2]) and nf == 0
+    for e in (0, 1, 3):
+        assert (b[e] != base[e]).mean() > 0.05
+    perm = [3, 1, 0, 2]
+    b2, m2, _, L2 = oracle_mod.grouped_project_lowrank(NV, base[perm], Bb[perm], Ab[perm], [ws2[p] for p in perm], aor)
+    assert np.array_equal(b2, b[perm]) and np.array_equal(m2, m[perm])
+    assert np.array_equal(L2.view(np.uint32), L[perm].view(np.uint32))
+    gm = rng.normal(0, 1, (E, N, G)).astype(np.float32)
+    dB, dA = oracle_mod.grouped_lowrank_grad(gm, Bb, Ab, aor)
+    gm2 = gm.copy()
+    gm2[1] *= 2.0                                                       # exact in fp32
+    dB2, dA2 = oracle_mod.grouped_lowrank_grad(gm2, Bb, Ab, aor)
+    assert np.array_equal(np.delete(dB2, 1, 0), np.delete(dB, 1, 0)) and np.array_equal(dB2[1], 2 * dB[1])
+    assert np.array_equal(np.delete(dA2, 1, 0), np.delete(dA, 1, 0)) and np.array_equal(dA2[1], 2 * dA[1])
