@@ -59,6 +59,9 @@ def lib():
         L.or_project_lowrank.argtypes = [ctypes.c_int, _i64, _i64, ctypes.c_int, ctypes.c_float, ctypes.c_float,
                                          _p, _p, _p, _p, _p, _p, _p]
         L.or_lowrank_grad.argtypes = [_i64, _i64, ctypes.c_int, ctypes.c_double, _p, _p, _p, _p, _p]
+        L.or_fit_scale_delta.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _p, _p, _p, _p, _p]
+        L.or_group_reduce.argtypes = [_i64, _i64, _i64, _p, _p]
+        L.or_project_group_delta.argtypes = [ctypes.c_int, _i64, _i64, _i64, ctypes.c_float, _p, _p, _p, _p, _p, _p]
         L.or_num_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -408,3 +411,55 @@ def grouped_lowrank_grad(gm, B_bits, A_bits, alpha_over_r):
     for e in range(E):
         dB[e], dA[e] = lowrank_grad(gm[e], B_bits[e], A_bits[e], alpha_over_r)
     return dB, dA
+
+
+# --- scale-family variants (ablation appendix) --------------------------------
+
+def fit_scale_delta(fmt, codes, scales, ws2, dW_bits):
+    """Least-squares code-preserving fit of a weight update dW [N, K] (bf16 bits):
+    per block delta = <c, dW> / <c, c> (0 for an all-zero code block). Returns
+    (delta, captured, total, latent): float64 [N, G] x 3 and the fp32 latent
+    fl32(s(byte) + fl32(delta)) (None when scales is None)."""
+    dW = _c(dW_bits, np.uint16)
+    codes = _c(codes, np.uint8)
+    N, K = dW.shape
+    G = K // BLOCK[fmt]
+    delta = np.empty((N, G), dtype=np.float64)
+    cap = np.empty((N, G), dtype=np.float64)
+    tot = np.empty((N, G), dtype=np.float64)
+    latent = None
+    sc = None
+    if scales is not None:
+        sc = _c(scales, np.uint8)
+        latent = np.empty((N, G), dtype=np.float32)
+    lib().or_fit_scale_delta(fmt, N, K, _ptr(codes), _ptr(sc), float(ws2), _ptr(dW), _ptr(delta), _ptr(cap),
+                             _ptr(tot), _ptr(latent))
+    return delta, cap, tot, latent
+
+
+def group_reduce(g, gd):
+    """Gradient of a per-group additive scale delta: the sum of each group's G / gd
+    consecutive block gradients, float64 [N, gd]."""
+    g = _c(g, np.float32)
+    N, G = g.shape
+    assert G % gd == 0
+    out = np.empty((N, gd), dtype=np.float64)
+    lib().or_group_reduce(N, G, int(gd), _ptr(g), _ptr(out))
+    return out
+
+
+def project_group_delta(fmt, base_scales, delta, ws2):
+    """Projection of fl32(s(base byte) + delta[n, b // (G / gd)]). Returns
+    (bytes, mask, nonfinite, latent)."""
+    base = _c(base_scales, np.uint8)
+    d = _c(delta, np.float32)
+    N, G = base.shape
+    gd = d.shape[1]
+    assert d.shape[0] == N and G % gd == 0
+    out = np.empty((N, G), dtype=np.uint8)
+    mask = np.empty((N, G), dtype=np.uint8)
+    latent = np.empty((N, G), dtype=np.float32)
+    nf = ctypes.c_int64(0)
+    lib().or_project_group_delta(fmt, N, G, int(gd), float(ws2), _ptr(base), _ptr(d), _ptr(out), _ptr(mask),
+                                 ctypes.byref(nf), _ptr(latent))
+    return out, mask, int(nf.value), latent

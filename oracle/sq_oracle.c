@@ -462,3 +462,76 @@ int or_num_threads(void) {
     return 1;
 #endif
 }
+
+/* ------------------------------------------------------------------ */
+/* Scale-family variants (ablation appendix)                           */
+/* ------------------------------------------------------------------ */
+
+/* Least-squares code-preserving fit of a weight-space update (the Spider
+ * paragraph of the ablations: "solve per block for the least-squares best
+ * code-preserving scale delta"). Within block b of row n the representable
+ * updates are t * c_b (c_b the block's E2M1 code values), so the fit is
+ *   delta[n,b] = <c_b, dW_b> / <c_b, c_b>,
+ * in absolute scale units (the update of the block's weights is c_b * delta).
+ * Reading: a block whose codes are all zero has no representable direction;
+ * its delta is 0. Also returned per block, when the arrays are given:
+ *   captured[n,b] = <c_b, dW_b>^2 / <c_b, c_b>   (|| projection ||^2, 0 for a zero block)
+ *   total[n,b]    = || dW_b ||^2
+ *   latent[n,b]   = fl32(scale(byte) + fl32(delta))   (the fitted scale, for the grid projection)
+ * dW is bf16 [N, K]; sums in float64, in element order. */
+void or_fit_scale_delta(int fmt, int64_t N, int64_t K, const uint8_t *codes, const uint8_t *scales, float ws2,
+                        const uint16_t *dW, double *delta, double *captured, double *total, float *latent) {
+  const int B = or_block(fmt);
+  const int64_t G = K / B;
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n) {
+    for (int64_t b = 0; b < G; ++b) {
+      double cw = 0.0, cc = 0.0, ww = 0.0;
+      for (int64_t k = b * B; k < (b + 1) * B; ++k) {
+        const double c = or_e2m1(or_code_nibble(codes, K, n, k));
+        const double w = or_bf16(dW[n * K + k]);
+        cw += c * w;
+        cc += c * c;
+        ww += w * w;
+      }
+      const double d = cc > 0.0 ? cw / cc : 0.0;
+      delta[n * G + b] = d;
+      if (captured) captured[n * G + b] = cc > 0.0 ? cw * cw / cc : 0.0;
+      if (total) total[n * G + b] = ww;
+      if (latent) latent[n * G + b] = or_scale_f32(fmt, ws2, scales[n * G + b]) + (float)d;
+    }
+  }
+}
+
+/* Granularity ladder (ablations, "Granularity alone over-perturbs"): a direct
+ * additive scale delta at granularity gd, one value per group of G / gd
+ * consecutive blocks of a row (gd = 1: one per row, PEQA; gd = G: per block).
+ * The latent of block b is s(byte) + delta[n, b / (G / gd)], so the gradient of
+ * a group delta is the sum of its blocks' (masked) scale gradients:
+ *   out[n, j] = sum_{b in group j} g[n, b]            (float64, block order) */
+void or_group_reduce(int64_t N, int64_t G, int64_t gd, const float *g, double *out) {
+  const int64_t W = G / gd;
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t j = 0; j < gd; ++j) {
+      double s = 0.0;
+      for (int64_t b = j * W; b < (j + 1) * W; ++b) s += (double)g[n * G + b];
+      out[n * gd + j] = s;
+    }
+}
+
+/* Projection of the group-delta latent fl32(s(byte) + delta[n, b / (G / gd)])
+ * (one fp32 add, the decoded scale of or_scale_f32) onto the grid. */
+void or_project_group_delta(int fmt, int64_t N, int64_t G, int64_t gd, float ws2, const uint8_t *base,
+                            const float *delta, uint8_t *bytes, uint8_t *mask, int64_t *nonfinite, float *latent) {
+  const int64_t W = G / gd;
+  int64_t nan_count = 0;
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t b = 0; b < G; ++b) {
+      const float L = or_scale_f32(fmt, ws2, base[n * G + b]) + delta[n * gd + b / W];
+      int is_nan = 0;
+      or_project_one(fmt, ws2, L, &bytes[n * G + b], &mask[n * G + b], &is_nan);
+      nan_count += is_nan;
+      if (latent) latent[n * G + b] = L;
+    }
+  *nonfinite = nan_count;
+}
