@@ -460,6 +460,49 @@ def adapter_leg(h, S, stream, reps=10):
     return out
 
 
+def variants_leg(h, S, pk, stream, reps=10):
+    """The scale-family variant kernels on the layer's largest plane (gate_proj,
+    14336 x 4096 NVFP4): the least-squares fit of a bf16 weight update (delta and both
+    energies out), the group gradient at gd = 4 and the group-delta projection at gd = 4.
+    Algorithmic bytes: fit 2 (dW) + 0.5 (codes) bytes per weight + 4 (delta) per block;
+    group gradient 4 per block in; projection 1 (base) + 1 + 1 + 4 (byte, mask, latent) per block."""
+    st = max(S.lin, key=lambda t: t["lin"].N * t["lin"].K)
+    l = st["lin"]
+    G = l.K // S.wl.block
+    gen = torch.Generator(device="cuda").manual_seed(404)
+    dW = (torch.randn(l.N, l.K, device="cuda", generator=gen) * 1e-4).to(torch.bfloat16)
+    delta = torch.empty(l.N, G, device="cuda")
+    cap, tot = torch.empty_like(delta), torch.empty_like(delta)
+    gd = 4
+    gdelta = torch.randn(l.N, gd, device="cuda", generator=gen) * st["ws2"] * 8
+    gout = torch.empty(l.N, gd, device="cuda")
+    qb = torch.empty(l.N, G, dtype=torch.uint8, device="cuda")
+    mask, lat = torch.empty_like(qb), torch.empty_like(delta)
+    blocks, weights = l.N * G, l.N * l.K
+    legs = (("fit", 2.5 * weights + 4 * blocks,
+             lambda: h.sq_fit_scale_delta(S.wl.fmt, st["codes"], dW, st["ws2"], want_energy=False, stream=stream)),
+            ("group_grad", 4 * blocks + 4 * l.N * gd, lambda: h.sq_group_reduce(st["g"], gd, out=gout, stream=stream)),
+            ("project_group_delta", 7 * blocks,
+             lambda: h.sq_project_group_delta(S.wl.fmt, st["base_scales"], gdelta, st["ws2"], bytes_out=qb,
+                                              mask_out=mask, latent_out=lat, stream=stream)))
+    out = {"plane": [l.N, l.K], "linear": l.name, "gd": gd}
+    for name, by, fn in legs:
+        for _ in range(3):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        out[name] = {"us": ms * 1e3, "bytes": int(by), "achieved": by / (ms / 1e3) / 1e9, "unit": "GB/s",
+                     "frac": by / (ms / 1e3) / 1e9 / pk["hbm_gbs"]}
+    h.sq_sync(stream)
+    return out
+
+
 def cublas_context(S, stream, steps=5):
     """torch.matmul (cuBLAS, bf16 in and out, fp32 accumulation) on pre-decoded weights
     for the same three contractions per linear: context for the fused kernels, which
@@ -614,6 +657,7 @@ def run_ours(args):
     if not args.no_context:
         context["plane_ceiling"] = plane_ceiling(h, pk, stream)
         context["adapter_kernels"] = adapter_leg(h, S, stream)
+        context["variant_kernels"] = variants_leg(h, S, pk, stream)
         context["cublas_context"] = cublas_context(S, stream)
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)

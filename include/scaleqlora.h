@@ -14,8 +14,10 @@
  *   sq_rollback        undo a merge with its on-grid delta (Sec. 5 Payoff 3)
  *   sq_swap_scales     scale-only hot-swap of the served adapter (Sec. 5)
  *   sq_count_diff      byte-level audit of two buffers (Sec. 5)
- *   sq_grouped_*       the contractions, projection and merge over the experts of an MoE
- *                      linear, one launch each (Sec. 3)
+ *   sq_grouped_*       the contractions, projection, merge and adapters over the experts of
+ *                      an MoE linear, one launch each (Sec. 3)
+ *   sq_fit_scale_delta, sq_group_reduce, sq_project_group_delta
+ *                      scale-family variants of the ablation appendix
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -220,6 +222,39 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
  * SQ_ERR_CUDA; there is no handle, so no error text. */
 sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
                                 const uint8_t *mask, float *g, int32_t *device_status, void *stream);
+
+/* ---------------------------------------------------------------- scale-family variants
+ * (ablation appendix; the same frozen codes, other reduction sets) */
+
+/* Least-squares code-preserving fit of a weight-space update dW (the Spider
+ * paragraph: the best per-block scale delta for a given update): block b of row n
+ * can only move by t * c (c its E2M1 code values), so
+ *   delta[n,b]    = <c, dW_b> / <c, c>      (0 for a block of zero codes)
+ *   captured[n,b] = <c, dW_b>^2 / <c, c>    (energy of the projection onto the block's codes)
+ *   total[n,b]    = ||dW_b||^2
+ *   latent[n,b]   = fl32(scale(byte) + delta)  (the fitted scale; project it with sq_project_scales)
+ * fp32 sums in element order. codes device [N, K/2]; dW device bf16 [N, K]; delta_out
+ * device fp32 [N, K/B]; captured_out, total_out, latent_out device fp32 [N, K/B] or NULL;
+ * scales device u8 [N, K/B], needed only with latent_out. K % 32 == 0. */
+sq_status sq_fit_scale_delta(sq_handle h, int32_t fmt, int64_t N, int64_t K, float ws2, const uint8_t *codes,
+                             const uint8_t *scales, const uint16_t *dW, float *delta_out, float *captured_out,
+                             float *total_out, float *latent_out, void *stream);
+
+/* Granularity ladder (ablation appendix, "Granularity alone over-perturbs"): a direct
+ * additive scale delta at granularity gd, one value per group of G / gd consecutive
+ * blocks of a row (gd = 1: per row, PEQA; gd = G: per block). The gradient of the
+ * group deltas is the sum of the group's (masked) block scale gradients:
+ *   out[n, j] = sum_{b in group j} g[n, b]     (fp32, block order)
+ * g device fp32 [N, G]; out device fp32 [N, gd]; gd >= 1 divides G. */
+sq_status sq_group_reduce(sq_handle h, int64_t N, int64_t G, int64_t gd, const float *g, float *out, void *stream);
+
+/* The group-delta latent fl32(scale(base byte) + delta[n, b / (G / gd)]) projected as
+ * sq_project_scales does (bytes, mask, NaN count), the latent optionally kept for
+ * sq_merge. base_scales device u8 [N, G]; delta device fp32 [N, gd]; bytes_out device
+ * u8 [N, G]; mask_out, latent_out or NULL; nonfinite device int32 or NULL. */
+sq_status sq_project_group_delta(sq_handle h, int32_t fmt, int64_t N, int64_t G, int64_t gd, float ws2,
+                                 const uint8_t *base_scales, const float *delta, uint8_t *bytes_out, uint8_t *mask_out,
+                                 int32_t *nonfinite, float *latent_out, void *stream);
 
 /* ---------------------------------------------------------------- experts
  * Mixture-of-experts layers (Sec. 3 "MoE: a batched grouped-expert kernel": the

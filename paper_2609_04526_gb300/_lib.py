@@ -29,7 +29,8 @@ EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_s
            "sq_scale_grad", "sq_project_scales", "sq_merge", "sq_project_lowrank", "sq_lowrank_grad",
            "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
            "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
-           "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad")
+           "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad", "sq_fit_scale_delta", "sq_group_reduce",
+           "sq_project_group_delta")
 
 
 class SQError(RuntimeError):
@@ -88,6 +89,9 @@ def load() -> ctypes.CDLL:
     L.sq_grouped_merge.argtypes = [vp, GW, vp, vp, vp, vp, vp]
     L.sq_grouped_project_lowrank.argtypes = [vp, GW, i32, f32, vp, vp, vp, vp, vp, vp, vp]
     L.sq_grouped_lowrank_grad.argtypes = [vp, i32, i64, i64, i32, f32, vp, vp, vp, vp, vp, vp]
+    L.sq_fit_scale_delta.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp]
+    L.sq_group_reduce.argtypes = [vp, i64, i64, i64, vp, vp, vp]
+    L.sq_project_group_delta.argtypes = [vp, i32, i64, i64, i64, f32, vp, vp, vp, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
@@ -370,3 +374,42 @@ class Handle:
         self._check(self._L.sq_grouped_lowrank_grad(self._h, E, N, G, r, alpha_over_r, _ptr(g), _ptr(B), _ptr(A),
                                                     _ptr(dB), _ptr(dA), _stream(stream)))
         return dB, dA
+
+
+    # scale-family variants -----------------------------------------------------
+    def sq_fit_scale_delta(self, fmt: int, codes: torch.Tensor, dW: torch.Tensor, ws2: float = 1.0,
+                           scales: Optional[torch.Tensor] = None, want_energy: bool = False, stream=None):
+        """Least-squares per-block scale delta of a bf16 weight update dW [N, K] against the
+        codes [N, K/2]. Returns (delta, captured, total, latent); the last three are None
+        unless asked for (energies with want_energy, the latent when scales are given)."""
+        N, K = dW.shape
+        G = K // BLOCK[fmt]
+        delta = torch.empty(N, G, dtype=torch.float32, device=dW.device)
+        cap = torch.empty_like(delta) if want_energy else None
+        tot = torch.empty_like(delta) if want_energy else None
+        lat = torch.empty_like(delta) if scales is not None else None
+        self._check(self._L.sq_fit_scale_delta(self._h, fmt, N, K, ws2, _ptr(codes), _ptr(scales), _ptr(dW),
+                                               _ptr(delta), _ptr(cap), _ptr(tot), _ptr(lat), _stream(stream)))
+        return delta, cap, tot, lat
+
+    def sq_group_reduce(self, g: torch.Tensor, gd: int, out: Optional[torch.Tensor] = None, stream=None):
+        """Gradient of per-group scale deltas: sums of each group's G / gd block gradients, [N, gd]."""
+        N, G = g.shape
+        if out is None:
+            out = torch.empty(N, gd, dtype=torch.float32, device=g.device)
+        self._check(self._L.sq_group_reduce(self._h, N, G, gd, _ptr(g), _ptr(out), _stream(stream)))
+        return out
+
+    def sq_project_group_delta(self, fmt: int, base_scales: torch.Tensor, delta: torch.Tensor, ws2: float,
+                               bytes_out: Optional[torch.Tensor] = None, mask_out: Optional[torch.Tensor] = None,
+                               nonfinite: Optional[torch.Tensor] = None, latent_out: Optional[torch.Tensor] = None,
+                               stream=None):
+        """Projection of s(base byte) + delta[n, b // (G / gd)]; delta [N, gd]. Returns (bytes, mask, latent)."""
+        N, G = base_scales.shape
+        gd = delta.shape[1]
+        if bytes_out is None:
+            bytes_out = torch.empty(N, G, dtype=torch.uint8, device=base_scales.device)
+        self._check(self._L.sq_project_group_delta(self._h, fmt, N, G, gd, ws2, _ptr(base_scales), _ptr(delta),
+                                                   _ptr(bytes_out), _ptr(mask_out), _ptr(nonfinite), _ptr(latent_out),
+                                                   _stream(stream)))
+        return bytes_out, mask_out, latent_out

@@ -741,6 +741,79 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
   SQ_GUARD_END
 }
 
+sq_status sq_fit_scale_delta(sq_handle h, int32_t fmt, int64_t N, int64_t K, float ws2, const uint8_t *codes,
+                             const uint8_t *scales, const uint16_t *dW, float *delta_out, float *captured_out,
+                             float *total_out, float *latent_out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_ws2(h, fmt, ws2));
+  if (N < 0 || N > kMaxDim || K < 0 || K % 32 != 0 || K > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "shape [%lld, %lld]: N in [0, 2^24], K a multiple of 32 in [0, 2^24]",
+                (long long)N, (long long)K);
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  if (N == 0 || K == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, codes, "codes"));
+  SQ_TRY(check_buf(h, dW, "dW"));
+  SQ_TRY(check_buf(h, delta_out, "delta_out"));
+  if (captured_out && !aligned16(captured_out)) return fail(h, SQ_ERR_INVALID_ARG, "captured_out must be 16-byte aligned");
+  if (total_out && !aligned16(total_out)) return fail(h, SQ_ERR_INVALID_ARG, "total_out must be 16-byte aligned");
+  if (latent_out) {
+    if (!aligned16(latent_out)) return fail(h, SQ_ERR_INVALID_ARG, "latent_out must be 16-byte aligned");
+    SQ_TRY(check_buf(h, scales, "scales (needed for latent_out)"));
+  }
+  cudaError_t e = sqi::launch_fit(fmt, N, K, ws2, codes, scales, dW, delta_out, captured_out, total_out, latent_out,
+                                  dev->sm_count, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "fit launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_group_reduce(sq_handle h, int64_t N, int64_t G, int64_t gd, const float *g, float *out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  if (gd < 1 || (G > 0 && (gd > G || G % gd != 0)))
+    return fail(h, SQ_ERR_INVALID_ARG, "gd=%lld must be >= 1 and divide G=%lld", (long long)gd, (long long)G);
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  if (N == 0 || G == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, g, "g"));
+  SQ_TRY(check_buf(h, out, "out"));
+  cudaError_t e = sqi::launch_group_reduce(N, G, gd, g, out, dev->sm_count, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "group reduction launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_project_group_delta(sq_handle h, int32_t fmt, int64_t N, int64_t G, int64_t gd, float ws2,
+                                 const uint8_t *base_scales, const float *delta, uint8_t *bytes_out, uint8_t *mask_out,
+                                 int32_t *nonfinite, float *latent_out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_plane(h, fmt, N, G, ws2));
+  if (gd < 1 || (G > 0 && (gd > G || G % gd != 0)))
+    return fail(h, SQ_ERR_INVALID_ARG, "gd=%lld must be >= 1 and divide G=%lld", (long long)gd, (long long)G);
+  if (nonfinite && (reinterpret_cast<uintptr_t>(nonfinite) & 3u))
+    return fail(h, SQ_ERR_INVALID_ARG, "nonfinite must be 4-byte aligned");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (N > 0 && G > 0) {
+    SQ_TRY(check_buf(h, base_scales, "base_scales"));
+    SQ_TRY(check_buf(h, delta, "delta"));
+    SQ_TRY(check_buf(h, bytes_out, "bytes_out"));
+    if (mask_out && !aligned16(mask_out)) return fail(h, SQ_ERR_INVALID_ARG, "mask_out must be 16-byte aligned");
+    if (latent_out && !aligned16(latent_out)) return fail(h, SQ_ERR_INVALID_ARG, "latent_out must be 16-byte aligned");
+  }
+  cudaError_t e = sqi::launch_project_group_delta(fmt, N, G, gd, ws2, base_scales, delta, bytes_out, mask_out,
+                                                  nonfinite, latent_out, dev->sm_count, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "group-delta projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
 sq_status sq_grouped_fwd(sq_handle h, const sq_grouped_weight *w, const int64_t *offsets, const uint16_t *X,
                          uint16_t *Y, void *stream) {
   if (!h) return SQ_ERR_INVALID_ARG;

@@ -112,6 +112,18 @@ cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r,
                                 cudaStream_t stream, int experts = 1);
 constexpr int kMaxLowRank = 256;  // r limit of the adapter kernels
 
+// Scale-family variants (ablation appendix): the least-squares code-preserving fit
+// of a weight update per block; the group gradient and the group-delta projection
+// of the granularity ladder (gd groups of G / gd blocks per row).
+cudaError_t launch_fit(int fmt, int64_t N, int64_t K, float ws2, const uint8_t *codes, const uint8_t *scales,
+                       const uint16_t *dW, float *delta, float *captured, float *total, float *latent, int sm_count,
+                       cudaStream_t stream);
+cudaError_t launch_group_reduce(int64_t N, int64_t G, int64_t gd, const float *g, float *out, int sm_count,
+                                cudaStream_t stream);
+cudaError_t launch_project_group_delta(int fmt, int64_t N, int64_t G, int64_t gd, float ws2, const uint8_t *base,
+                                       const float *delta, uint8_t *bytes_out, uint8_t *mask_out, int32_t *nonfinite,
+                                       float *latent_out, int sm_count, cudaStream_t stream);
+
 // Device-side error codes written to the error word.
 constexpr int kErrWaitTimeout = 1;
 

@@ -552,6 +552,162 @@ __global__ void __launch_bounds__(kThreads) sq_adapter_reduce_kernel(int64_t cou
   }
 }
 
+// ---------------------------------------------------------------- scale-family variants
+//
+// Least-squares code-preserving fit (ablation appendix, the Spider paragraph): the
+// updates a block can represent are multiples t * c of its code values c, so the
+// best scale delta for a weight update dW is <c, dW> / <c, c> (0 for a block of
+// zero codes), in absolute scale units. One thread per block; the block's codes
+// and bf16 update are contiguous (B / 2 and 2 B bytes), so a warp reads whole
+// segments. fp32 sums in element order: c * dW, c * c and dW * dW are exact (E2M1
+// values have two significant bits, bf16 eight), the sums round.
+
+// E2M1 nibble -> fp32 from the format's fields: sign bit 3, exponent bits 1-2
+// (bias 1), mantissa bit 0; exponent 0 is the subnormal 0 or 0.5.
+__device__ __forceinline__ float e2m1_value(uint32_t nib) {
+  const uint32_t e = (nib >> 1) & 3u, m = nib & 1u;
+  const uint32_t mag = e == 0 ? (m ? 0x3F000000u : 0u) : (((126u + e) << 23) | (m << 22));
+  return __uint_as_float(mag | ((nib & 8u) << 28));
+}
+
+template <int FMT>
+__device__ __forceinline__ void fit_one(int64_t i, float ws2, const uint32_t (&cw32)[(FMT == 0 ? 16 : 32) / 8],
+                                        const uint4 (&w4)[(FMT == 0 ? 16 : 32) / 8],
+                                        const uint8_t *__restrict__ scales, float *__restrict__ delta,
+                                        float *__restrict__ captured, float *__restrict__ total,
+                                        float *__restrict__ latent) {
+  constexpr int B = FMT == 0 ? 16 : 32;
+  float cwsum = 0.f, ccsum = 0.f, wwsum = 0.f;
+#pragma unroll
+  for (int q = 0; q < B / 8; ++q) {
+    const uint32_t wv[4] = {w4[q].x, w4[q].y, w4[q].z, w4[q].w};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float c = e2m1_value((cw32[q] >> (4 * j)) & 0xFu);
+      const float w = __uint_as_float(j & 1 ? wv[j >> 1] & 0xFFFF0000u : wv[j >> 1] << 16);
+      // the products are exact in fp32 (at most 2 + 8 or 8 + 8 significant bits), so a
+      // fused multiply-add rounds exactly as the product followed by the sum
+      cwsum = __fmaf_rn(c, w, cwsum);
+      ccsum = __fmaf_rn(c, c, ccsum);
+      wwsum = __fmaf_rn(w, w, wwsum);
+    }
+  }
+  const float d = ccsum > 0.f ? __fdiv_rn(cwsum, ccsum) : 0.f;
+  delta[i] = d;
+  if (captured) captured[i] = ccsum > 0.f ? __fdiv_rn(__fmul_rn(cwsum, cwsum), ccsum) : 0.f;
+  if (total) total[i] = wwsum;
+  if (latent) latent[i] = __fadd_rn(scale_value<FMT>(scales[i], ws2), d);
+}
+
+// Each thread fits blocks i and i + stride per iteration, so the loads of both are in
+// flight before either is reduced.
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_fit_kernel(int64_t blocks, float ws2, const uint8_t *__restrict__ codes,
+                                                          const uint8_t *__restrict__ scales,
+                                                          const uint16_t *__restrict__ dW, float *__restrict__ delta,
+                                                          float *__restrict__ captured, float *__restrict__ total,
+                                                          float *__restrict__ latent) {
+  constexpr int B = FMT == 0 ? 16 : 32;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < blocks; i += 2 * stride) {
+    const int64_t i2 = i + stride;
+    const bool two = i2 < blocks;
+    uint32_t ca[B / 8], cb[B / 8];
+    uint4 wa[B / 8], wb[B / 8];
+#pragma unroll
+    for (int q = 0; q < B / 8; ++q) {
+      ca[q] = __ldg(reinterpret_cast<const uint32_t *>(codes + i * (B / 2)) + q);
+      wa[q] = __ldcs(reinterpret_cast<const uint4 *>(dW + i * B) + q);
+      if (two) {
+        cb[q] = __ldg(reinterpret_cast<const uint32_t *>(codes + i2 * (B / 2)) + q);
+        wb[q] = __ldcs(reinterpret_cast<const uint4 *>(dW + i2 * B) + q);
+      }
+    }
+    fit_one<FMT>(i, ws2, ca, wa, scales, delta, captured, total, latent);
+    if (two) fit_one<FMT>(i2, ws2, cb, wb, scales, delta, captured, total, latent);
+  }
+}
+
+// Granularity ladder (ablation appendix): one additive scale delta per group of
+// W = G / gd consecutive blocks of a row. Its gradient is the sum of the group's
+// block gradients. One warp per group: lane l sums blocks l, l + 32, ... in order
+// (coalesced loads), then a fixed butterfly of shuffles adds the 32 partial sums,
+// so the result is the same on every run.
+__global__ void __launch_bounds__(kThreads) sq_group_reduce_kernel(int64_t groups, int64_t W,
+                                                                   const float *__restrict__ g,
+                                                                   float *__restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5); t < groups; t += warps) {
+    const float *src = g + t * W;
+    float s = 0.f;
+    for (int64_t b = lane; b < W; b += 32) s = __fadd_rn(s, __ldg(src + b));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xFFFFFFFFu, s, o));
+    if (lane == 0) out[t] = s;
+  }
+}
+
+// The group-delta latent fl32(s(base byte) + delta[n, b / W]) projected onto the grid
+// (the a5 device code), with mask, NaN count and the latent itself for the merge.
+// 16 consecutive blocks per thread (16-byte loads and stores, as the projection);
+// the row and group of each block are stepped along, since a vector may cross rows.
+template <int FMT>
+__device__ __forceinline__ void project_group_one(int64_t n, int64_t b, int64_t gd, int64_t W, float ws2, float cap,
+                                                  uint32_t base_byte, const float *__restrict__ delta, uint32_t &by,
+                                                  uint32_t &mk, uint32_t &na, float &L) {
+  L = __fadd_rn(scale_value<FMT>(base_byte, ws2), __ldg(delta + n * gd + b / W));
+  project_one<FMT>(L, ws2, cap, by, mk, na);
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_project_group_delta_kernel(
+    int64_t N, int64_t G, int64_t W, float ws2, float cap, const uint8_t *__restrict__ base,
+    const float *__restrict__ delta, uint8_t *__restrict__ bytes_out, uint8_t *__restrict__ mask_out,
+    int32_t *__restrict__ nonfinite, float *__restrict__ latent_out) {
+  const int64_t count = N * G, gd = G / W, nvec = count / 16;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  uint32_t nan_count = 0;
+  for (int64_t v = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; v < nvec; v += stride) {
+    const uint4 b4 = __ldcs(reinterpret_cast<const uint4 *>(base) + v);
+    const uint32_t bw[4] = {b4.x, b4.y, b4.z, b4.w};
+    int64_t n = (16 * v) / G, b = 16 * v - n * G;
+    uint32_t ob[4] = {0, 0, 0, 0}, om[4] = {0, 0, 0, 0};
+    float L[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      uint32_t by, mk, na;
+      project_group_one<FMT>(n, b, gd, W, ws2, cap, (bw[i >> 2] >> (8 * (i & 3))) & 0xFFu, delta, by, mk, na, L[i]);
+      ob[i >> 2] |= by << (8 * (i & 3));
+      om[i >> 2] |= mk << (8 * (i & 3));
+      nan_count += na;
+      if (++b == G) {
+        b = 0;
+        ++n;
+      }
+    }
+    __stcs(reinterpret_cast<uint4 *>(bytes_out) + v, make_uint4(ob[0], ob[1], ob[2], ob[3]));
+    if (mask_out) __stcs(reinterpret_cast<uint4 *>(mask_out) + v, make_uint4(om[0], om[1], om[2], om[3]));
+    if (latent_out) {
+      float4 *dst = reinterpret_cast<float4 *>(latent_out) + 4 * v;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) __stcs(dst + q, make_float4(L[4 * q], L[4 * q + 1], L[4 * q + 2], L[4 * q + 3]));
+    }
+  }
+  // ragged tail (< 16 blocks) by the first threads of block 0
+  if (blockIdx.x == 0 && threadIdx.x < count - nvec * 16) {
+    const int64_t i = nvec * 16 + threadIdx.x, n = i / G, b = i - n * G;
+    uint32_t by, mk, na;
+    float L;
+    project_group_one<FMT>(n, b, gd, W, ws2, cap, base[i], delta, by, mk, na, L);
+    bytes_out[i] = static_cast<uint8_t>(by);
+    if (mask_out) mask_out[i] = static_cast<uint8_t>(mk);
+    if (latent_out) latent_out[i] = L;
+    nan_count += na;
+  }
+  if (nonfinite) warp_add_i32(nonfinite, nan_count);
+}
+
 // Contraction chunks for an output of `tiles` 64 x 64 tiles: enough CTAs for about
 // two per SM, chunks of at least 4 steps.
 int64_t adapter_chunks(int64_t kdim, int64_t tiles, int sm_count) {
@@ -691,6 +847,52 @@ cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r,
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+cudaError_t launch_fit(int fmt, int64_t N, int64_t K, float ws2, const uint8_t *codes, const uint8_t *scales,
+                       const uint16_t *dW, float *delta, float *captured, float *total, float *latent, int sm_count,
+                       cudaStream_t stream) {
+  const int64_t blocks = N * (K / (fmt == 0 ? 16 : 32));
+  if (blocks == 0) return cudaSuccess;
+  // two blocks per thread and iteration; up to eight CTAs per SM keep enough loads in flight
+  const int64_t want = (blocks + 2 * kThreads - 1) / (2 * kThreads), cap = static_cast<int64_t>(sm_count) * 8;
+  const unsigned grid = static_cast<unsigned>(want < cap ? want : cap);
+  if (fmt == 0)
+    sq_fit_kernel<0><<<grid, kThreads, 0, stream>>>(blocks, ws2, codes, scales, dW, delta, captured, total, latent);
+  else
+    sq_fit_kernel<1><<<grid, kThreads, 0, stream>>>(blocks, ws2, codes, scales, dW, delta, captured, total, latent);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_reduce(int64_t N, int64_t G, int64_t gd, const float *g, float *out, int sm_count,
+                                cudaStream_t stream) {
+  const int64_t groups = N * gd;
+  if (groups == 0) return cudaSuccess;
+  const int64_t per = kThreads / 32;  // one warp per group
+  const int64_t want = (groups + per - 1) / per, cap = static_cast<int64_t>(sm_count) * 8;
+  sq_group_reduce_kernel<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, 0, stream>>>(groups, G / gd, g,
+                                                                                                   out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_project_group_delta(int fmt, int64_t N, int64_t G, int64_t gd, float ws2, const uint8_t *base,
+                                       const float *delta, uint8_t *bytes_out, uint8_t *mask_out, int32_t *nonfinite,
+                                       float *latent_out, int sm_count, cudaStream_t stream) {
+  if (nonfinite) {
+    cudaError_t e = cudaMemsetAsync(nonfinite, 0, sizeof(int32_t), stream);
+    if (e != cudaSuccess) return e;
+  }
+  const int64_t count = N * G;
+  if (count == 0) return cudaSuccess;
+  const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
+  const unsigned grid = grid_for(count, sm_count);
+  if (fmt == 0)
+    sq_project_group_delta_kernel<0><<<grid, kThreads, 0, stream>>>(N, G, G / gd, ws2, cap, base, delta, bytes_out,
+                                                                    mask_out, nonfinite, latent_out);
+  else
+    sq_project_group_delta_kernel<1><<<grid, kThreads, 0, stream>>>(N, G, G / gd, ws2, cap, base, delta, bytes_out,
+                                                                    mask_out, nonfinite, latent_out);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_rollback(int fmt, int64_t count, float ws2, const float *delta, uint8_t *scales_inout,
