@@ -62,6 +62,9 @@ def lib():
         L.or_fit_scale_delta.argtypes = [ctypes.c_int, _i64, _i64, _p, _p, ctypes.c_float, _p, _p, _p, _p, _p]
         L.or_group_reduce.argtypes = [_i64, _i64, _i64, _p, _p]
         L.or_project_group_delta.argtypes = [ctypes.c_int, _i64, _i64, _i64, ctypes.c_float, _p, _p, _p, _p, _p, _p]
+        L.or_control_weight.argtypes = [_i64, _i64, _p, _p, _p]
+        L.or_control_grad.argtypes = [_i64, _i64, _i64, _p, _p, _p, _p]
+        L.or_lowrank_product.argtypes = [_i64, _i64, ctypes.c_int, ctypes.c_double, _p, _p, _p]
         L.or_num_threads.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -463,3 +466,37 @@ def project_group_delta(fmt, base_scales, delta, ws2):
     lib().or_project_group_delta(fmt, N, G, int(gd), float(ws2), _ptr(base), _ptr(d), _ptr(out), _ptr(mask),
                                  ctypes.byref(nf), _ptr(latent))
     return out, mask, int(nf.value), latent
+
+
+def control_weight(W_bits, dS):
+    """W' = bf16(fl32(W * fl32(1 + dS[n, k // 16]))) of the multiplicative control, float64 [N, K]."""
+    W = _c(W_bits, np.uint16)
+    d = _c(dS, np.float32)
+    N, K = W.shape
+    assert d.shape == (N, K // 16)
+    out = np.empty((N, K), dtype=np.float64)
+    lib().or_control_weight(N, K, _ptr(W), _ptr(d), _ptr(out))
+    return out
+
+
+def control_grad_f64(W_bits, X, dY):
+    """g[n, b] = sum over the block's columns of W[n, k] (dY^T X)[n, k], float64 [N, K/16]."""
+    W = _c(W_bits, np.uint16)
+    X = _c(X, np.float64)
+    dY = _c(dY, np.float64)
+    M, K = X.shape
+    N = dY.shape[1]
+    g = np.empty((N, K // 16), dtype=np.float64)
+    lib().or_control_grad(M, N, K, _ptr(W), _ptr(X), _ptr(dY), _ptr(g))
+    return g
+
+
+def lowrank_product(B_bits, A_bits, alpha_over_r):
+    """(alpha/r) B A in float64 from bf16 bits B [N, r], A [r, G]."""
+    B = _c(B_bits, np.uint16)
+    A = _c(A_bits, np.uint16)
+    N, r = B.shape
+    G = A.shape[1]
+    out = np.empty((N, G), dtype=np.float64)
+    lib().or_lowrank_product(N, G, r, float(alpha_over_r), _ptr(B), _ptr(A), _ptr(out))
+    return out

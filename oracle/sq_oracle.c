@@ -535,3 +535,65 @@ void or_project_group_delta(int fmt, int64_t N, int64_t G, int64_t gd, float ws2
     }
   *nonfinite = nan_count;
 }
+
+/* Full-precision multiplicative control (ablation appendix: unquantized bf16
+ * weights, the within-block pattern frozen, one coefficient per (row, block of 16),
+ * W' = W (1 + dS[o, g(i)])). Reading of the arithmetic: the factor is
+ * f = fl32(1 + dS), the product is rounded to fp32 and then to bf16 (round to
+ * nearest, ties to even), i.e. W' = bf16(fl32(W * f)); the contractions then use
+ * W' like any decoded weight. */
+static float or_round_bf16(float x) {
+  uint32_t u;
+  memcpy(&u, &x, 4);
+  if ((u & 0x7F800000u) == 0x7F800000u) {  /* inf or NaN: keep (quiet NaN) */
+    if (u & 0x007FFFFFu) u |= 0x00400000u;
+    u &= 0xFFFF0000u;
+  } else {
+    const uint32_t lsb = (u >> 16) & 1u;
+    u = (u + 0x7FFFu + lsb) & 0xFFFF0000u;  /* round half to even at bit 16 */
+  }
+  float r;
+  memcpy(&r, &u, 4);
+  return r;
+}
+
+void or_control_weight(int64_t N, int64_t K, const uint16_t *W, const float *dS, double *Wp) {
+  const int64_t G = K / 16;
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k) {
+      const float f = 1.0f + dS[n * G + k / 16];
+      const float w = (float)or_bf16(W[n * K + k]);
+      Wp[n * K + k] = (double)or_round_bf16(w * f);
+    }
+}
+
+/* Gradient of L with respect to dS[o, b] through W' = W (1 + dS) (the rounding of
+ * W' passed straight through): sum over the block's columns of W[o,i] dW[o,i],
+ * dW = dY^T X, float64. X [M, K], dY [M, N] as float64. */
+void or_control_grad(int64_t M, int64_t N, int64_t K, const uint16_t *W, const double *X, const double *dY,
+                     double *g) {
+  const int64_t G = K / 16;
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t b = 0; b < G; ++b) {
+      double s = 0.0;
+      for (int64_t k = b * 16; k < (b + 1) * 16; ++k) {
+        double dw = 0.0;
+        for (int64_t m = 0; m < M; ++m) dw += dY[m * N + n] * X[m * K + k];
+        s += or_bf16(W[n * K + k]) * dw;
+      }
+      g[n * G + b] = s;
+    }
+}
+
+/* The control's low-rank coefficient plane dS = (alpha/r) B A (float64), B [N, r],
+ * A [r, G] bf16. */
+void or_lowrank_product(int64_t N, int64_t G, int r, double alpha_over_r, const uint16_t *B, const uint16_t *A,
+                        double *out) {
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t b = 0; b < G; ++b) {
+      double s = 0.0;
+      for (int j = 0; j < r; ++j) s += or_bf16(B[n * r + j]) * or_bf16(A[(int64_t)j * G + b]);
+      out[n * G + b] = alpha_over_r * s;
+    }
+}

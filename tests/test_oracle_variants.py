@@ -16,6 +16,12 @@ Granularity ladder (a per-group additive scale delta, gd groups per row):
   gd = 1 the row sums;
 - the group-delta latent is numpy's fp32 s + delta; zero delta returns every finite
   base byte; in range the byte is torch's E4M3 cast of latent / ws2.
+
+Full-precision multiplicative control (W' = W (1 + dS) per row and block of 16):
+- W' equals numpy's fp32 factor and product followed by torch's bf16 cast, and W for
+  dS = 0;
+- the coefficient gradient equals central differences of the (unrounded) bilinear
+  form sum(dY * X W'^T); the low-rank coefficient plane equals numpy's (alpha/r) B A.
 """
 import numpy as np
 import torch
@@ -152,3 +158,51 @@ def test_group_delta_projection(oracle_mod):
     cast = torch.from_numpy(np.where(inrange, q, 1.0).astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8)
     assert np.array_equal(b[inrange], cast.numpy()[inrange])
     assert (b != base).mean() > 0.3
+
+
+def test_control_weight_rounding(oracle_mod):
+    """W' against numpy: fp32 factor 1 + dS, fp32 product, torch's bf16 (RNE) cast.
+    dS = 0 returns W exactly; a product just above a bf16 midpoint rounds up."""
+    rng = np.random.default_rng(80)
+    N, K = 6, 64
+    Wb, W64 = _bf16_bits(rng.normal(0, 0.05, (N, K)))
+    dS = (rng.normal(0, 0.1, (N, K // 16))).astype(np.float32)
+    Wp = oracle_mod.control_weight(Wb, dS)
+    f = (np.float32(1.0) + dS).astype(np.float32)
+    prod = (W64.astype(np.float32) * np.repeat(f, 16, axis=1)).astype(np.float32)
+    ref = torch.from_numpy(prod).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(Wp, ref)
+    assert np.array_equal(oracle_mod.control_weight(Wb, np.zeros_like(dS)), W64)
+    # w = 1 + 2^-7 (bf16), f = 1 + 2^-8: 1 + 1.5 * 2^-7 + 2^-15 lies just above a midpoint -> 1 + 2^-6
+    Wt, _ = _bf16_bits(np.full((1, 16), 1 + 2 ** -7))
+    out = oracle_mod.control_weight(Wt, np.full((1, 1), 2 ** -8, np.float32))
+    assert (out == 1 + 2 ** -6).all()
+
+
+def test_control_gradient_is_the_derivative_of_the_bilinear_form(oracle_mod):
+    """L(dS) = sum(dY * X (W (1 + dS))^T) is linear in dS (unrounded W'), so its central
+    differences (numpy) equal g for every block."""
+    rng = np.random.default_rng(81)
+    M, N, K = 5, 4, 48
+    Wb, W64 = _bf16_bits(rng.normal(0, 0.05, (N, K)))
+    X = rng.normal(0, 1, (M, K))
+    dY = rng.normal(0, 1, (M, N))
+    g = oracle_mod.control_grad_f64(Wb, X, dY)
+
+    def L(dS):
+        Wp = W64 * (1 + np.repeat(dS, 16, axis=1))
+        return float(np.sum(dY * (X @ Wp.T)))
+
+    for n in range(N):
+        for b in range(K // 16):
+            E = np.zeros((N, K // 16))
+            E[n, b] = 0.5
+            fd = (L(E) - L(-E)) / 1.0
+            assert abs(fd - g[n, b]) <= 1e-12 * (1 + np.abs(g).max())
+
+
+def test_lowrank_product_matches_numpy(oracle_mod):
+    rng = np.random.default_rng(82)
+    Bb, B64 = _bf16_bits(rng.normal(0, 1, (9, 5)))
+    Ab, A64 = _bf16_bits(rng.normal(0, 1, (5, 7)))
+    assert np.allclose(oracle_mod.lowrank_product(Bb, Ab, 0.75), 0.75 * (B64 @ A64), rtol=1e-14, atol=1e-14)
