@@ -486,6 +486,33 @@ def variants_leg(h, S, pk, stream, reps=10):
              lambda: h.sq_project_group_delta(S.wl.fmt, st["base_scales"], gdelta, st["ws2"], bytes_out=qb,
                                               mask_out=mask, latent_out=lat, stream=stream)))
     out = {"plane": [l.N, l.K], "linear": l.name, "gd": gd}
+    # the full-precision multiplicative control on the same linear: W the bf16 decoded
+    # weight, one coefficient per (row, block of 16); its three contractions, TFLOP/s
+    Wbf = predecoded_weight(S.wl, st)
+    dS = torch.randn(l.N, l.K // 16, device="cuda", generator=gen) * 0.05
+    X = S.acts[l.x]
+    Yc = torch.empty(S.wl.M, l.N, dtype=torch.bfloat16, device="cuda")
+    dXc = torch.empty(S.wl.M, l.K, dtype=torch.bfloat16, device="cuda")
+    gc = torch.empty(l.N, l.K // 16, device="cuda")
+    flops = 2 * S.wl.M * l.N * l.K
+    ctl = {"shape": [S.wl.M, l.N, l.K]}
+    for name, fn in (("fwd", lambda: h.sq_control_fwd(Wbf, dS, X, Y=Yc, stream=stream)),
+                     ("dx", lambda: h.sq_control_bwd_dx(Wbf, dS, st["dY"], dX=dXc, stream=stream)),
+                     ("grad", lambda: h.sq_control_grad(Wbf, X, st["dY"], g=gc, stream=stream))):
+        for _ in range(2):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        ctl[name] = {"ms": ms, "achieved": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s",
+                     "frac": flops / (ms / 1e3) / 1e12 / pk["bf16_sustained"]}
+    out["control"] = ctl
+    del Wbf, Yc, dXc
     for name, by, fn in legs:
         for _ in range(3):
             fn()

@@ -16,8 +16,8 @@
  *   sq_count_diff      byte-level audit of two buffers (Sec. 5)
  *   sq_grouped_*       the contractions, projection, merge and adapters over the experts of
  *                      an MoE linear, one launch each (Sec. 3)
- *   sq_fit_scale_delta, sq_group_reduce, sq_project_group_delta
- *                      scale-family variants of the ablation appendix
+ *   sq_fit_scale_delta, sq_group_reduce, sq_project_group_delta, sq_control_*,
+ *   sq_lowrank_product scale-family variants of the ablation appendix
  * with W[n,k] = code[n,k] * s[n, k / B] decoded on the fly, where (Sec. 2)
  *   NVFP4: B = 16, s = E4M3(scale byte) * ws2 (fp32 tensor scale)
  *   MXFP4: B = 32, s = E8M0(scale byte) = 2^(byte - 127), ws2 must be 1.0
@@ -255,6 +255,40 @@ sq_status sq_group_reduce(sq_handle h, int64_t N, int64_t G, int64_t gd, const f
 sq_status sq_project_group_delta(sq_handle h, int32_t fmt, int64_t N, int64_t G, int64_t gd, float ws2,
                                  const uint8_t *base_scales, const float *delta, uint8_t *bytes_out, uint8_t *mask_out,
                                  int32_t *nonfinite, float *latent_out, void *stream);
+
+/* Full-precision multiplicative control (ablation appendix: on unquantized bf16
+ * weights the within-block pattern is frozen and one coefficient per (row, block of
+ * 16) is learned, W' = W (1 + dS[o, i / 16]); no codes, no grid, no STE). Arithmetic:
+ * f = fl32(1 + dS), W' = bf16(fl32(W * f)) rounded to nearest even, then the
+ * contractions of sq_fwd / sq_bwd_dx with W' (bf16 operands, fp32 accumulation). */
+typedef struct {
+  int32_t N;            /* out features, N % 8 == 0                          */
+  int32_t K;            /* in features, K % 32 == 0                          */
+  const uint16_t *W;    /* device bf16 [N, K], frozen                        */
+  const float *dS;      /* device fp32 [N, K/16] coefficients (FWD, DX)      */
+} sq_control_weight;
+
+/* Y = X W'^T. X device bf16 [M, K]; Y device bf16 [M, N]. */
+sq_status sq_control_fwd(sq_handle h, const sq_control_weight *w, const uint16_t *X, int64_t M, uint16_t *Y,
+                         void *stream);
+
+/* dX = dY W'. dY device bf16 [M, N]; dX device bf16 [M, K]. */
+sq_status sq_control_bwd_dx(sq_handle h, const sq_control_weight *w, const uint16_t *dY, int64_t M, uint16_t *dX,
+                            void *stream);
+
+/* Coefficient gradient through W' = W (1 + dS) (its bf16 rounding passed straight
+ * through): g[o, b] = sum_{i in block b} W[o, i] (dY^T X)[o, i], the dW tile reduced
+ * on chip as in sq_scale_grad. g device fp32 [N, K/16]; dS is not read; M == 0
+ * gives zeros. */
+sq_status sq_control_grad(sq_handle h, const sq_control_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
+                          float *g, void *stream);
+
+/* The control's low-rank coefficient plane: out = alpha_over_r * B A, B [N, r] and
+ * A [r, G] bf16, out device fp32 [N, G], fp32 sums in a fixed order (the same on
+ * every run); its gradients are sq_lowrank_grad of the coefficient gradient. Uses
+ * the handle's scratch. 1 <= r <= 256. */
+sq_status sq_lowrank_product(sq_handle h, int64_t N, int64_t G, int32_t r, float alpha_over_r, const uint16_t *B,
+                             const uint16_t *A, float *out, void *stream);
 
 /* ---------------------------------------------------------------- experts
  * Mixture-of-experts layers (Sec. 3 "MoE: a batched grouped-expert kernel": the

@@ -30,7 +30,7 @@ EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_s
            "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
            "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
            "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad", "sq_fit_scale_delta", "sq_group_reduce",
-           "sq_project_group_delta")
+           "sq_project_group_delta", "sq_control_fwd", "sq_control_bwd_dx", "sq_control_grad", "sq_lowrank_product")
 
 
 class SQError(RuntimeError):
@@ -47,6 +47,10 @@ class _SqWeight(ctypes.Structure):
 class _SqGroupedWeight(ctypes.Structure):
     _fields_ = [("fmt", ctypes.c_int32), ("E", ctypes.c_int32), ("N", ctypes.c_int32), ("K", ctypes.c_int32),
                 ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("ws2", ctypes.POINTER(ctypes.c_float))]
+
+
+class _SqControlWeight(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int32), ("K", ctypes.c_int32), ("W", ctypes.c_void_p), ("dS", ctypes.c_void_p)]
 
 
 _lib = None
@@ -92,6 +96,11 @@ def load() -> ctypes.CDLL:
     L.sq_fit_scale_delta.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp, vp, vp, vp]
     L.sq_group_reduce.argtypes = [vp, i64, i64, i64, vp, vp, vp]
     L.sq_project_group_delta.argtypes = [vp, i32, i64, i64, i64, f32, vp, vp, vp, vp, vp, vp, vp]
+    CW = ctypes.POINTER(_SqControlWeight)
+    L.sq_control_fwd.argtypes = [vp, CW, vp, i64, vp, vp]
+    L.sq_control_bwd_dx.argtypes = [vp, CW, vp, i64, vp, vp]
+    L.sq_control_grad.argtypes = [vp, CW, vp, vp, i64, vp, vp]
+    L.sq_lowrank_product.argtypes = [vp, i64, i64, i32, f32, vp, vp, vp, vp]
     for name in EXPORTS:
         if name not in ("sq_status_string", "sq_last_error"):
             getattr(L, name).restype = ctypes.c_int
@@ -413,3 +422,47 @@ class Handle:
                                                    _ptr(bytes_out), _ptr(mask_out), _ptr(nonfinite), _ptr(latent_out),
                                                    _stream(stream)))
         return bytes_out, mask_out, latent_out
+
+    # full-precision multiplicative control -------------------------------------
+    def sq_control_fwd(self, W: torch.Tensor, dS: torch.Tensor, X: torch.Tensor, Y: Optional[torch.Tensor] = None,
+                       stream=None):
+        """Y = X W'^T with W' = bf16(W (1 + dS)) per row and block of 16; W [N, K] bf16, dS [N, K/16]."""
+        N, K = W.shape
+        M = X.shape[0]
+        if Y is None:
+            Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+        cw = _SqControlWeight(N, K, _ptr(W), _ptr(dS))
+        self._check(self._L.sq_control_fwd(self._h, ctypes.byref(cw), _ptr(X), M, _ptr(Y), _stream(stream)))
+        return Y
+
+    def sq_control_bwd_dx(self, W: torch.Tensor, dS: torch.Tensor, dY: torch.Tensor,
+                          dX: Optional[torch.Tensor] = None, stream=None):
+        N, K = W.shape
+        M = dY.shape[0]
+        if dX is None:
+            dX = torch.empty(M, K, dtype=torch.bfloat16, device=dY.device)
+        cw = _SqControlWeight(N, K, _ptr(W), _ptr(dS))
+        self._check(self._L.sq_control_bwd_dx(self._h, ctypes.byref(cw), _ptr(dY), M, _ptr(dX), _stream(stream)))
+        return dX
+
+    def sq_control_grad(self, W: torch.Tensor, X: torch.Tensor, dY: torch.Tensor, g: Optional[torch.Tensor] = None,
+                        stream=None):
+        """Coefficient gradient g[o, b] = sum over the block of W[o, i] (dY^T X)[o, i], [N, K/16]."""
+        N, K = W.shape
+        M = X.shape[0]
+        if g is None:
+            g = torch.empty(N, K // 16, dtype=torch.float32, device=X.device)
+        cw = _SqControlWeight(N, K, _ptr(W), None)
+        self._check(self._L.sq_control_grad(self._h, ctypes.byref(cw), _ptr(X), _ptr(dY), M, _ptr(g), _stream(stream)))
+        return g
+
+    def sq_lowrank_product(self, B: torch.Tensor, A: torch.Tensor, alpha_over_r: float,
+                           out: Optional[torch.Tensor] = None, stream=None):
+        """(alpha/r) B A, B [N, r] and A [r, G] bf16 -> fp32 [N, G]."""
+        N, r = B.shape
+        G = A.shape[1]
+        if out is None:
+            out = torch.empty(N, G, dtype=torch.float32, device=B.device)
+        self._check(self._L.sq_lowrank_product(self._h, N, G, r, alpha_over_r, _ptr(B), _ptr(A), _ptr(out),
+                                               _stream(stream)))
+        return out

@@ -227,6 +227,55 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   return SQ_OK;
 }
 
+// ------------------------------------------------------------------ multiplicative control
+
+sq_status check_control(sq_handle h, const sq_control_weight *w, bool need_dS) {
+  if (!w) return fail(h, SQ_ERR_INVALID_ARG, "control weight is NULL");
+  if (w->N <= 0 || w->N % 8 != 0 || w->N > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "N=%d must be positive, a multiple of 8 and <= 2^24", w->N);
+  if (w->K <= 0 || w->K % 32 != 0 || w->K > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "K=%d must be positive, a multiple of 32 and <= 2^24", w->K);
+  if (!w->W || !aligned16(w->W)) return fail(h, SQ_ERR_INVALID_ARG, "W must be non-NULL and 16-byte aligned");
+  if (need_dS && (!w->dS || !aligned16(w->dS)))
+    return fail(h, SQ_ERR_INVALID_ARG, "dS must be non-NULL and 16-byte aligned");
+  return SQ_OK;
+}
+
+// One control contraction: FWD a = X, out = Y; DX a = dY, out = dX; SGRAD a = dY, b = X, out = g.
+sq_status run_control(sq_handle h, int mode, const sq_control_weight *w, const void *a_ptr, const void *b_ptr,
+                      int64_t M, void *out, cudaStream_t stream) {
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  CUtensorMap tmA, tmB, tmOut;
+  if (mode == sqi::MODE_FWD) {
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->K, M, 64, sqi::kBM));
+    SQ_TRY(make_act_map(h, &tmB, w->W, w->K, w->N, 64, 128));  // W [N, K] in 64 x 128 boxes
+    SQ_TRY(make_out_map(h, &tmOut, out, w->N, M));
+  } else if (mode == sqi::MODE_DX) {
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kBM));
+    SQ_TRY(make_act_map(h, &tmB, w->W, w->K, w->N, 64, 128));
+    SQ_TRY(make_out_map(h, &tmOut, out, w->K, M));
+  } else {
+    SQ_TRY(make_act_map(h, &tmA, a_ptr, w->N, M, 64, sqi::kSgradBK));
+    SQ_TRY(make_act_map(h, &tmB, b_ptr, w->K, M, 64, sqi::kSgradBK));
+  }
+  sqi::GemmArgs a;
+  a.mode = mode;
+  a.fmt = 2;
+  a.M = M;
+  a.N = w->N;
+  a.K = w->K;
+  a.codes = reinterpret_cast<const uint8_t *>(w->W);
+  a.scales = reinterpret_cast<const uint8_t *>(w->dS);
+  a.ws2 = 1.0f;
+  a.out = out;
+  a.mask = nullptr;
+  a.err = dev->err_word;
+  cudaError_t e = sqi::launch_control(a, tmA, tmB, mode == sqi::MODE_SGRAD ? nullptr : &tmOut, dev->sm_count, stream);
+  if (e != cudaSuccess) return cuda_fail(h, e, "control kernel launch");
+  return SQ_OK;
+}
+
 // ------------------------------------------------------------------ grouped (experts)
 
 constexpr int kMaxExperts = 1 << 16;
@@ -810,6 +859,75 @@ sq_status sq_project_group_delta(sq_handle h, int32_t fmt, int64_t N, int64_t G,
   cudaError_t e = sqi::launch_project_group_delta(fmt, N, G, gd, ws2, base_scales, delta, bytes_out, mask_out,
                                                   nonfinite, latent_out, dev->sm_count, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "group-delta projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_control_fwd(sq_handle h, const sq_control_weight *w, const uint16_t *X, int64_t M, uint16_t *Y,
+                         void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_control(h, w, true));
+  SQ_TRY(check_tokens(h, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, Y, "Y"));
+  return run_control(h, sqi::MODE_FWD, w, X, nullptr, M, Y, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_control_bwd_dx(sq_handle h, const sq_control_weight *w, const uint16_t *dY, int64_t M, uint16_t *dX,
+                            void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_control(h, w, true));
+  SQ_TRY(check_tokens(h, M));
+  if (M == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, dY, "dY"));
+  SQ_TRY(check_buf(h, dX, "dX"));
+  return run_control(h, sqi::MODE_DX, w, dY, nullptr, M, dX, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_control_grad(sq_handle h, const sq_control_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
+                          float *g, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_control(h, w, false));
+  SQ_TRY(check_tokens(h, M));
+  SQ_TRY(check_buf(h, g, "g"));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (M == 0) {
+    DeviceState *dev = nullptr;
+    SQ_TRY(ensure_device(h, &dev));
+    cudaError_t e = cudaMemsetAsync(g, 0, static_cast<size_t>(w->N) * (w->K / 16) * sizeof(float), st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(g)");
+    return SQ_OK;
+  }
+  SQ_TRY(check_buf(h, X, "X"));
+  SQ_TRY(check_buf(h, dY, "dY"));
+  return run_control(h, sqi::MODE_SGRAD, w, dY, X, M, g, st);
+  SQ_GUARD_END
+}
+
+sq_status sq_lowrank_product(sq_handle h, int64_t N, int64_t G, int32_t r, float alpha_over_r, const uint16_t *B,
+                             const uint16_t *A, float *out, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  if (N < 0 || G < 0 || N > kMaxDim || G > kMaxDim)
+    return fail(h, SQ_ERR_INVALID_ARG, "plane shape [%lld, %lld] out of range", (long long)N, (long long)G);
+  if (r < 1 || r > sqi::kMaxLowRank) return fail(h, SQ_ERR_INVALID_ARG, "rank r=%d must be in [1, 256]", r);
+  if (!std::isfinite(alpha_over_r)) return fail(h, SQ_ERR_INVALID_ARG, "alpha_over_r must be finite");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  if (N == 0 || G == 0) return SQ_OK;
+  SQ_TRY(check_buf(h, B, "B"));
+  SQ_TRY(check_buf(h, A, "A"));
+  SQ_TRY(check_buf(h, out, "out"));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_product_workspace(N, G, r, dev->sm_count)));
+  cudaError_t e = sqi::launch_lowrank_product(N, G, r, alpha_over_r, B, A, out, static_cast<float *>(dev->workspace),
+                                              dev->sm_count, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "low-rank product launch");
   return SQ_OK;
   SQ_GUARD_END
 }

@@ -353,6 +353,11 @@ __device__ __forceinline__ uint32_t scale_bf16x2(uint32_t byte) {
 
 // ------------------------------------------------------------- shared pieces
 
+// Weight formats of the contraction kernels: NVFP4 (0) and MXFP4 (1) codes with
+// block scales, and the full-precision multiplicative control of the ablation
+// appendix (2): bf16 weights W times fl32(1 + dS) per (row, block of 16).
+constexpr int kFmtBf16Mul = 2;
+
 struct KParams {
   const uint8_t *codes;
   const uint8_t *scales;
@@ -726,6 +731,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           mbar_drain(&afull[i % SA], static_cast<uint32_t>(i / SA) & 1u);
       }
     }
+  } else if (FMT == kFmtBf16Mul && warp == C::kCodeWarp) {
+    // ------------------------------------------------------ bf16 weight TMA (both CTAs)
+    // The multiplicative control: this CTA's half of the bf16 weight tile goes
+    // straight into the decoded-weight slot (two 64-wide boxes, 128-byte swizzle:
+    // the layout the MMAs read), once the MMAs of the slot's previous use are done;
+    // the decode warps then scale it in place. cfull[s] counts its bytes.
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      int e = 0;
+      for (int tile = cluster; tile < total && ok; tile += nclusters) {
+        int tm, tn;
+        resolve_tile<GR>(p, tile, e, tm, tn);
+        const int32_t half0 = tn * C::kTile + 128 * static_cast<int32_t>(rank);
+        for (int kb = 0; kb < num_k; ++kb, ++it) {
+          const int s = it % S;
+          const uint32_t use = static_cast<uint32_t>(it / S);
+          if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+          mbar_arrive_expect_tx(&cfull[s], C::kB);
+          for (int j = 0; j < 2; ++j) {
+            if (MODE == MODE_FWD)  // 128 weight rows (out features) x 64 k
+              tma_load_2d(smem_u32(ring_b(s)) + j * 16384, &tmC, &cfull[s], kb * C::kBK + 64 * j, half0);
+            else                   // 128 contraction rows x 64 k-columns
+              tma_load_2d(smem_u32(ring_b(s)) + j * 16384, &tmC, &cfull[s], half0 + 64 * j, kb * C::kBK);
+          }
+        }
+      }
+      if (*abort_flag) {
+        for (int i = (it > S ? it - S : 0); i < it; ++i) mbar_drain(&cfull[i % S], static_cast<uint32_t>(i / S) & 1u);
+      }
+    }
   } else if (warp == C::kCodeWarp) {
     // ------------------------------------------------------ code TMA (both CTAs)
     if (lane == 0) {
@@ -825,6 +861,75 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         if (!mbar_spin(&afull[(2 * it) % SA], static_cast<uint32_t>((2 * it) / SA) & 1u, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
+      }
+    }
+  } else if (FMT == kFmtBf16Mul && warp >= C::kEpiWarps) {
+    // ------------------------------------------------------ in-place scaling (both CTAs)
+    // Each thread scales its 32-weight unit of the landed bf16 tile: W' =
+    // bf16(fl32(W * f)) with f = fl32(1 + dS[n, k / 16]) per block of 16, rounded
+    // to nearest even, written back in place; factors are loaded one stage ahead.
+    const int dw = warp - C::kEpiWarps;
+    const int u = dw * 32 + lane;
+    const int row = (u & 7) + 8 * (u >> 5), quarter = (u >> 3) & 3;
+    uint32_t b_off[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int chunk = 4 * (quarter & 1) + c;
+      b_off[c] = MODE == MODE_FWD
+                     ? (quarter >> 1) * 16384 + (row >> 3) * 1024 + (row & 7) * 128 + ((chunk ^ (row & 7)) << 4)
+                     : (quarter >> 1) * 16384 + row * 128 + ((chunk ^ (row & 7)) << 4);
+    }
+    const float *dS = reinterpret_cast<const float *>(p.scales);
+    const int64_t G = p.K / 16;
+    auto factors = [&](int tile, int kb, int tn, float &f0, float &f1) {
+      f0 = f1 = 0.f;
+      if (tile >= total) return;
+      int64_t n, k;
+      pair_unit_coords<MODE>(u, static_cast<int64_t>(tn) * C::kTile + 128 * rank, kb, n, k);
+      if (n >= p.N || k >= p.K) return;  // outside the weight: the tile holds zeros there
+      f0 = __fadd_rn(1.0f, __ldg(dS + n * G + k / 16));
+      f1 = __fadd_rn(1.0f, __ldg(dS + n * G + k / 16 + 1));
+    };
+    const uint32_t sink_addr = mapa_shared(smem_u32(&sink[rank * C::kDecWarps + dw]), 0);
+    int it = 0, s = 0, e = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int tile = cluster; tile < total && ok; tile += nclusters) {
+      int tm, tn;
+      resolve_tile<GR>(p, tile, e, tm, tn);
+      float f0, f1;
+      factors(tile, 0, tn, f0, f1);
+      for (int kb = 0; kb < num_k && ok; ++kb, ++it) {
+        float g0, g1;
+        factors(tile, kb + 1 < num_k ? kb + 1 : num_k, tn, g0, g1);  // next stage's factors
+        if (lane == 0) ok = mbar_wait(&cfull[s], ph, abort_flag, p.err);
+        ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+        __syncwarp();
+        if (!ok) break;
+        const uint32_t b_base = smem_u32(ring_b(s));
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const uint4 v = lds128(b_base + b_off[c]);
+          const float f = c < 2 ? f0 : f1;
+          const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+          uint32_t o[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(__fmul_rn(__uint_as_float(wv[q] << 16), f),
+                                                            __fmul_rn(__uint_as_float(wv[q] & 0xFFFF0000u), f));
+            o[q] = *reinterpret_cast<const uint32_t *>(&h2);
+          }
+          st_shared_v4(b_base + b_off[c], o[0], o[1], o[2], o[3]);
+        }
+        fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
+        __syncwarp();
+        if (lane == 0) st_async_signal(sink_addr, mapa_shared(smem_u32(&pready[s]), 0));
+        f0 = g0;
+        f1 = g1;
+        if (++s == S) {
+          s = 0;
+          ph ^= 1u;
+        }
       }
     }
   } else if (warp >= C::kEpiWarps) {
@@ -1052,7 +1157,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
                          const KParams p) {
   using C = SgradPairCfg;
   constexpr int S = C::kStages;
-  constexpr int B = FMT == 0 ? 16 : 32;
+  constexpr int B = FMT == 1 ? 32 : 16;  // the multiplicative control has one factor per 16 weights
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + S * C::kStageBytes);
@@ -1192,7 +1297,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
     for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
       int tm, tn;
       resolve_tile<GR, kSgradGroup>(p, tile, e, tm, tn);
-      // the expert's code plane, gradient plane and mask
+      // the expert's code plane (the multiplicative control: its bf16 weights), gradient plane and mask
       const uint8_t *codes = GR ? p.codes + e * p.N * (p.K / 2) : p.codes;
       float *g = static_cast<float *>(p.out) + (GR ? e * p.N * G : 0);
       const uint8_t *mask = p.mask ? p.mask + (GR ? e * p.N * G : 0) : nullptr;
@@ -1214,13 +1319,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
         }
         const int64_t k = col0 + c0;
         if (n >= p.N || k >= p.K) continue;
-        const uint4 cw = __ldg(reinterpret_cast<const uint4 *>(codes + n * (p.K / 2) + k / 2));
+        uint4 cw = make_uint4(0, 0, 0, 0);
+        if (FMT != kFmtBf16Mul) cw = __ldg(reinterpret_cast<const uint4 *>(codes + n * (p.K / 2) + k / 2));
         const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
         float part[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-          uint32_t o[4];
-          e2m1x8_to_bf16(words[c], o);
+          uint32_t o[4];  // 8 weights of the row as bf16 pairs: decoded codes, or the control's bf16 W
+          if (FMT == kFmtBf16Mul) {
+            const uint4 wq = __ldg(reinterpret_cast<const uint4 *>(codes + (n * p.K + k + 8 * c) * 2));
+            o[0] = wq.x;
+            o[1] = wq.y;
+            o[2] = wq.z;
+            o[3] = wq.w;
+          } else {
+            e2m1x8_to_bf16(words[c], o);
+          }
           float acc = 0.f;
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -1229,7 +1343,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
           }
           part[c] = acc;
         }
-        if (FMT == 0) {
+        if (FMT != 1) {
           const int64_t b = k / 16;
           float g0 = part[0] + part[1];
           float g1 = part[2] + part[3];

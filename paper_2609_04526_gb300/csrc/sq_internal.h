@@ -72,6 +72,18 @@ struct GroupedArgs {
 // packed codes as one [E * N, K/2] tensor (MODE_FWD / MODE_DX; unused for MODE_SGRAD).
 cudaError_t launch_grouped(const GroupedArgs &a, const CUtensorMap &tmCodes, int sm_count, cudaStream_t stream);
 
+// The contractions of the full-precision multiplicative control (a.fmt ignored):
+// a.codes is the bf16 weight W [N, K], a.scales the fp32 coefficients dS [N, K/16];
+// tmB the descriptor of W in 64 x 128 boxes with the 128-byte swizzle (FWD / DX),
+// or of X (SGRAD, as launch_gemm).
+cudaError_t launch_control(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB,
+                           const CUtensorMap *tmOut, int sm_count, cudaStream_t stream);
+// out = alpha_over_r * B A (B [N, r], A [r, G] bf16), through `workspace`
+// (lowrank_product_workspace bytes): the control's low-rank coefficient plane.
+size_t lowrank_product_workspace(int64_t N, int64_t G, int r, int sm_count);
+cudaError_t launch_lowrank_product(int64_t N, int64_t G, int r, float alpha_over_r, const uint16_t *B,
+                                   const uint16_t *A, float *out, float *workspace, int sm_count, cudaStream_t stream);
+
 // Launch one contraction. tmA is the TMA descriptor of the streamed bf16
 // activations; tmB that of the packed codes (MODE_FWD / MODE_DX) or of the second
 // bf16 operand (MODE_SGRAD); tmOut that of the bf16 output (MODE_FWD / MODE_DX:

@@ -455,6 +455,19 @@ struct DaRight {  // g[n = k][b = i]
   __device__ DaRight expert(int64_t e) const { return DaRight{g + e * estride, G, estride}; }
 };
 
+struct DsLeft {  // B[n = i][j = k] (the control's coefficient plane dS = (alpha/r) B A)
+  const uint16_t *B;
+  int64_t r, estride;
+  __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(B[i * r + k]); }
+  __device__ DsLeft expert(int64_t e) const { return DsLeft{B + e * estride, r, estride}; }
+};
+struct DsRight {  // A[j = k][b = i]
+  const uint16_t *A;
+  int64_t G, estride;
+  __device__ float operator()(int64_t i, int64_t k) const { return bf16_bits(A[k * G + i]); }
+  __device__ DsRight expert(int64_t e) const { return DsRight{A + e * estride, G, estride}; }
+};
+
 // partial[e][c][i][j] = sum_{k in chunk c} L_e(i, k) R_e(j, k), i < rows, j < cols,
 // for expert e = blockIdx.z / chunks and chunk c = blockIdx.z % chunks.
 template <class LeftT, class RightT, bool LEFT_K_FAST, bool RIGHT_K_FAST>
@@ -892,6 +905,32 @@ cudaError_t launch_project_group_delta(int fmt, int64_t N, int64_t G, int64_t gd
   else
     sq_project_group_delta_kernel<1><<<grid, kThreads, 0, stream>>>(N, G, G / gd, ws2, cap, base, delta, bytes_out,
                                                                     mask_out, nonfinite, latent_out);
+  return cudaGetLastError();
+}
+
+size_t lowrank_product_workspace(int64_t N, int64_t G, int r, int sm_count) {
+  const int64_t tiles = ((N + kT - 1) / kT) * ((G + kT - 1) / kT);
+  return static_cast<size_t>(adapter_chunks(r, tiles, sm_count) * N * G) * sizeof(float);
+}
+
+cudaError_t launch_lowrank_product(int64_t N, int64_t G, int r, float alpha_over_r, const uint16_t *B,
+                                   const uint16_t *A, float *out, float *workspace, int sm_count,
+                                   cudaStream_t stream) {
+  const int64_t tiles = ((N + kT - 1) / kT) * ((G + kT - 1) / kT);
+  const int64_t c = adapter_chunks(r, tiles, sm_count);
+  const int64_t kc = ((r + c - 1) / c + kKStep - 1) / kKStep * kKStep;
+  const int64_t chunks = (r + kc - 1) / kc;
+  const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT),
+                  static_cast<unsigned>(chunks));
+  // rows n, columns b, contraction j: B is j-contiguous, A is b-contiguous
+  sq_adapter_product_kernel<DsLeft, DsRight, true, false><<<grid, kThreads, 0, stream>>>(
+      N, G, r, kc, chunks, DsLeft{B, r, 0}, DsRight{A, G, 0}, workspace);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t count = N * G;
+  const unsigned cap = static_cast<unsigned>(sm_count) * kCtasPerSm;
+  const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((count + kThreads - 1) / kThreads, cap));
+  sq_adapter_reduce_kernel<<<blocks, kThreads, 0, stream>>>(count, 1, chunks, alpha_over_r, workspace, out);
   return cudaGetLastError();
 }
 

@@ -164,3 +164,98 @@ def test_variants_invalid_args(h):
         with pytest.raises(pkg.SQError) as ei:
             call()
         assert ei.value.status == -1, i
+
+
+def _control_inputs(M, N, K, seed, ds_scale=0.05):
+    gen = torch.Generator(device="cuda").manual_seed(seed)
+    W = (torch.randn(N, K, device="cuda", generator=gen) * 0.02).to(torch.bfloat16)
+    dS = torch.randn(N, K // 16, device="cuda", generator=gen) * ds_scale
+    X = torch.randn(M, K, device="cuda", generator=gen).to(torch.bfloat16)
+    dY = (torch.randn(M, N, device="cuda", generator=gen) * 1e-3).to(torch.bfloat16)
+    return W, dS, X, dY
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 392, 608), (64, 256, 512), (1, 8, 32), (1030, 264, 2080)])
+def test_control_parity_small(h, M, N, K):
+    """The multiplicative control's forward, input gradient and coefficient gradient
+    against the oracle (W' rounded as the oracle rounds it, contractions in float64)."""
+    W, dS, X, dY = _control_inputs(M, N, K, seed=M + N + K)
+    Y = h.sq_control_fwd(W, dS, X)
+    dX = h.sq_control_bwd_dx(W, dS, dY)
+    g = h.sq_control_grad(W, X, dY)
+    h.sq_sync()
+    Wp = oracle.control_weight(hbits(W), host(dS))
+    assert_close(f64(Y), oracle.fwd_f64(f64(X), Wp), what="Y")
+    assert_close(f64(dX), oracle.dx_f64(f64(dY), Wp), what="dX")
+    assert_close(host(g), oracle.control_grad_f64(hbits(W), f64(X), f64(dY)), what="g")
+
+
+def test_control_full_size_sampled(h):
+    """8192 x 14336 x 4096 (the c3 shape): sampled Y and dX elements and whole rows of
+    g against the oracle."""
+    M, N, K = 8192, 14336, 4096
+    W, dS, X, dY = _control_inputs(M, N, K, seed=9)
+    Y = h.sq_control_fwd(W, dS, X)
+    dX = h.sq_control_bwd_dx(W, dS, dY)
+    g = h.sq_control_grad(W, X, dY)
+    h.sq_sync()
+    rng = np.random.default_rng(9)
+    ns = np.unique(np.concatenate([[0, N - 1], rng.integers(0, N, 24)]))
+    ks = np.unique(np.concatenate([[0, K - 1], rng.integers(0, K, 24)]))
+    ms = np.unique(np.concatenate([[0, M - 1], rng.integers(0, M, 48)]))
+    Wp_rows = oracle.control_weight(hbits(W)[ns], host(dS)[ns])
+    Xm = f64(X[torch.from_numpy(ms).cuda()])
+    assert_close(f64(Y)[np.ix_(ms, ns)], Xm @ Wp_rows.T, what="Y samples")
+    Wp_all = oracle.control_weight(hbits(W), host(dS))
+    dYm = f64(dY[torch.from_numpy(ms).cuda()])
+    assert_close(f64(dX)[np.ix_(ms, ks)], dYm @ Wp_all[:, ks], what="dX samples")
+    rg = oracle.control_grad_f64(hbits(W)[ns], f64(X), f64(dY)[:, ns])
+    assert_close(host(g)[ns], rg, what="g rows")
+
+
+def test_control_adapter_chain(h):
+    """The control's low-rank coefficients dS = (alpha/r) B A -> forward -> coefficient
+    gradient -> adapter gradients, against the oracle chain; the product repeats."""
+    M, N, K, r = 300, 264, 512, 16
+    gen = torch.Generator(device="cuda").manual_seed(31)
+    W, _, X, dY = _control_inputs(M, N, K, seed=31)
+    B = (torch.randn(N, r, device="cuda", generator=gen) * 0.05).to(torch.bfloat16)
+    A = (torch.randn(r, K // 16, device="cuda", generator=gen) * 0.05).to(torch.bfloat16)
+    aor = 2.0
+    dS = h.sq_lowrank_product(B, A, aor)
+    dS2 = h.sq_lowrank_product(B, A, aor)
+    Y = h.sq_control_fwd(W, dS, X)
+    g = h.sq_control_grad(W, X, dY)
+    dB, dA = h.sq_lowrank_grad(g, B, A, aor)
+    h.sq_sync()
+    assert torch.equal(dS, dS2)
+    assert_close(host(dS), oracle.lowrank_product(hbits(B), hbits(A), aor), what="dS")
+    Wp = oracle.control_weight(hbits(W), host(dS))
+    assert_close(f64(Y), oracle.fwd_f64(f64(X), Wp), what="Y")
+    rg = oracle.control_grad_f64(hbits(W), f64(X), f64(dY))
+    assert_close(host(g), rg, what="g")
+    rdB, rdA = oracle.lowrank_grad(rg.astype(np.float32), hbits(B), hbits(A), aor)
+    assert_close(host(dB), rdB, what="dB")
+    assert_close(host(dA), rdA, what="dA")
+
+
+def test_control_invalid_args(h):
+    import paper_2609_04526_gb300 as pkg
+    W = torch.zeros(8, 32, dtype=torch.bfloat16, device="cuda")
+    dS = torch.zeros(8, 2, device="cuda")
+    X = torch.zeros(4, 32, dtype=torch.bfloat16, device="cuda")
+    bad = [
+        lambda: h.sq_control_fwd(torch.zeros(12, 32, dtype=torch.bfloat16, device="cuda"), dS, X),     # N % 8
+        lambda: h.sq_control_fwd(torch.zeros(8, 48, dtype=torch.bfloat16, device="cuda"), dS, X),      # K % 32
+        lambda: h.sq_lowrank_product(torch.zeros(8, 300, dtype=torch.bfloat16, device="cuda"),
+                                     torch.zeros(300, 2, dtype=torch.bfloat16, device="cuda"), 1.0),  # r > 256
+    ]
+    for call in bad:
+        with pytest.raises(pkg.SQError) as ei:
+            call()
+        assert ei.value.status == -1
+    Y = h.sq_control_fwd(W, dS, torch.zeros(0, 32, dtype=torch.bfloat16, device="cuda"))
+    g = h.sq_control_grad(W, torch.zeros(0, 32, dtype=torch.bfloat16, device="cuda"),
+                          torch.zeros(0, 8, dtype=torch.bfloat16, device="cuda"), g=torch.full((8, 2), 3.0, device="cuda"))
+    h.sq_sync()
+    assert Y.shape == (0, 8) and (g == 0).all()
