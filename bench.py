@@ -693,8 +693,8 @@ def run_ours(args):
         import oracle
         oracle.lib()
         host = host_copies(S, list(wl.linears))
-        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=256, n_dx=256,
-                                              n_rows=oracle.num_threads(), n_plane=1 << 17)
+        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=1024, n_dx=1024,
+                                              n_rows=6 * oracle.num_threads(), n_plane=1 << 18)
         cpu = {"value": flops_step / t_full / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
                "sample": desc, "sample_seconds": round(t_spent, 2), "extrapolated_step_seconds": round(t_full, 1)}
 
