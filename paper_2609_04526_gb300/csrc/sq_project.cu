@@ -341,11 +341,13 @@ __global__ void __launch_bounds__(kThreads) sq_swap_or_diff_kernel(int64_t count
 // follow expert e - 1's, and grid z (with the contraction chunk for the products)
 // selects the expert; a dense call is the case E = 1.
 // The three adapter kernels are register-tiled fp32 CUDA-core products: a CTA of 256
-// threads owns a 64 x 64 output tile, its operands staged in shared memory as fp32,
-// and each thread accumulates a 4 x 4 sub-tile (rows ty*4 .. +3, columns tx + 16c),
-// so 8 shared-memory loads feed 16 fused multiply-adds. Every output is summed
-// sequentially over the contraction index, so results do not change between runs.
-constexpr int kT = 64;  // output tile edge
+// threads owns a 64 x 64 output tile, its operands staged in shared memory as fp32
+// (contraction index outermost), and each thread accumulates a 4 x 4 sub-tile (rows
+// ty*4 .. +3, columns tx*4 .. +3), so two 16-byte shared-memory loads feed 16 fused
+// multiply-adds. Every output is summed sequentially over the contraction index, so
+// results do not change between runs.
+constexpr int kT = 64;   // output tile edge
+constexpr int kTP = 68;  // padded row of a staged operand (16-byte multiple; spreads the transposed stores)
 
 __device__ __forceinline__ float bf16_bits(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
 
@@ -356,8 +358,8 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
     uint8_t *__restrict__ bytes_out, uint8_t *__restrict__ mask_out, int32_t *__restrict__ nonfinite,
     float *__restrict__ latent_out) {
   extern __shared__ float lr_smem[];
-  float *sB = lr_smem;            // [kT rows][r]
-  float *sA = lr_smem + kT * r;   // [r][kT columns]
+  float *sB = lr_smem;             // [r][kTP]: B[n0 + row][j] at j * kTP + row
+  float *sA = lr_smem + kTP * r;   // [r][kT columns]
   const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kT;
   const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kT;
   // expert blockIdx.z: its planes, factors and (NVFP4 experts) tensor scale
@@ -373,8 +375,9 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
     cap = 448.0f * ws2;  // the same IEEE fp32 product as the host's single-plane cap
   }
   for (int i = threadIdx.x; i < kT * r; i += kThreads) {
-    const int64_t n = n0 + i / r;
-    sB[i] = n < N ? bf16_bits(B[n * r + i % r]) : 0.f;
+    const int row = i / r, j = i % r;
+    const int64_t n = n0 + row;
+    sB[j * kTP + row] = n < N ? bf16_bits(B[n * r + j]) : 0.f;
   }
   for (int i = threadIdx.x; i < r * kT; i += kThreads) {
     const int64_t b = b0 + i % kT;
@@ -388,11 +391,9 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[q][c] = 0.f;
   for (int j = 0; j < r; ++j) {
-    float bv[4], av[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) bv[q] = sB[(ty * 4 + q) * r + j];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) av[c] = sA[j * kT + tx + 16 * c];
+    const float4 b4 = *reinterpret_cast<const float4 *>(sB + j * kTP + ty * 4);
+    const float4 a4 = *reinterpret_cast<const float4 *>(sA + j * kT + tx * 4);
+    const float bv[4] = {b4.x, b4.y, b4.z, b4.w}, av[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q)
 #pragma unroll
@@ -403,7 +404,7 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
   for (int q = 0; q < 4; ++q) {
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      const int64_t n = n0 + ty * 4 + q, b = b0 + tx + 16 * c;
+      const int64_t n = n0 + ty * 4 + q, b = b0 + tx * 4 + c;
       if (n < N && b < G) {
         const int64_t i = n * G + b;
         const float L = fmaf(aor, acc[q][c], scale_value<FMT>(base[i], ws2));
@@ -474,8 +475,8 @@ template <class LeftT, class RightT, bool LEFT_K_FAST, bool RIGHT_K_FAST>
 __global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t rows, int64_t cols, int64_t kdim,
                                                                       int64_t kchunk, int64_t chunks, LeftT left_all,
                                                                       RightT right_all, float *__restrict__ partial) {
-  __shared__ float sl[2][kKStep][kT + 1];  // [buffer][k][i]
-  __shared__ float sr[2][kKStep][kT + 1];  // [buffer][k][j]
+  __shared__ __align__(16) float sl[2][kKStep][kTP];  // [buffer][k][i]
+  __shared__ __align__(16) float sr[2][kKStep][kTP];  // [buffer][k][j]
   const int64_t expert = blockIdx.z / chunks, chunk = blockIdx.z % chunks;
   const LeftT left = left_all.expert(expert);
   const RightT right = right_all.expert(expert);
@@ -523,11 +524,9 @@ __global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t ro
     if (more) load(k0 + kKStep);  // in flight while this step computes
 #pragma unroll
     for (int kk = 0; kk < kKStep; ++kk) {
-      float lv[4], rv[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) lv[q] = sl[buf][kk][ty * 4 + q];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) rv[c] = sr[buf][kk][tx + 16 * c];
+      const float4 l4 = *reinterpret_cast<const float4 *>(&sl[buf][kk][ty * 4]);
+      const float4 r4 = *reinterpret_cast<const float4 *>(&sr[buf][kk][tx * 4]);
+      const float lv[4] = {l4.x, l4.y, l4.z, l4.w}, rv[4] = {r4.x, r4.y, r4.z, r4.w};
 #pragma unroll
       for (int q = 0; q < 4; ++q)
 #pragma unroll
@@ -544,7 +543,7 @@ __global__ void __launch_bounds__(kThreads) sq_adapter_product_kernel(int64_t ro
   for (int q = 0; q < 4; ++q)
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      const int64_t i = i0 + ty * 4 + q, j = j0 + tx + 16 * c;
+      const int64_t i = i0 + ty * 4 + q, j = j0 + tx * 4 + c;
       if (i < rows && j < cols) out[i * cols + j] = acc[q][c];
     }
 }
@@ -796,7 +795,7 @@ cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float w
   const float cap = 448.0f * ws2;  // one IEEE fp32 multiply
   const dim3 grid(static_cast<unsigned>((N + kT - 1) / kT), static_cast<unsigned>((G + kT - 1) / kT),
                   static_cast<unsigned>(experts));
-  const size_t smem = static_cast<size_t>(2 * kT) * r * sizeof(float);  // <= 128 KiB for r <= 256
+  const size_t smem = static_cast<size_t>(kTP + kT) * r * sizeof(float);  // <= 132 KiB for r <= 256
   cudaError_t e;
   if (fmt == 0) {
     if ((e = cudaFuncSetAttribute(sq_project_lowrank_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
