@@ -103,3 +103,71 @@ def test_binding_refuses_to_fall_back(tmp_path, monkeypatch):
     monkeypatch.setattr(L, "_lib", None)
     with pytest.raises(ImportError):
         L.load()
+
+
+def _gw(fmt=0, E=3, N=64, K=128, codes=A16, scales=A16, ws2=(0.01, 0.02, 0.03)):
+    L = pkg._lib
+    arr = None if ws2 is None else (ctypes.c_float * len(ws2))(*ws2)
+    w = L._SqGroupedWeight(fmt, E, N, K, codes, scales,
+                           None if arr is None else ctypes.cast(arr, ctypes.POINTER(ctypes.c_float)))
+    return w, arr
+
+
+def _off(vals):
+    return (ctypes.c_int64 * len(vals))(*vals)
+
+
+def test_grouped_validation(built):
+    """Grouped calls reject bad experts, tensor scales and token layouts before any
+    device work; an empty batch is a no-op."""
+    h = pkg.Handle()
+    vp = ctypes.c_void_p
+    good_off = _off([0, 4, 4, 9])
+    cases = [
+        (_gw(E=0, ws2=()), good_off, "E=0"),
+        (_gw(ws2=None), good_off, "ws2"),                                   # NVFP4 needs ws2[E]
+        (_gw(ws2=(0.01, float("inf"), 0.03)), good_off, "ws2[1]"),
+        (_gw(fmt=1, ws2=(1.0, 0.5, 1.0)), good_off, "MXFP4"),
+        (_gw(N=12), good_off, "N=12"),
+        (_gw(K=48), good_off, "K=48"),
+        (_gw(codes=A16 + 4), good_off, "codes"),
+        (_gw(), _off([1, 4, 4, 9]), "offsets[0]"),
+        (_gw(), _off([0, 4, 3, 9]), "non-decreasing"),
+        (_gw(E=40000, N=65536, ws2=[1.0] * 40000), _off([0] * 40000 + [8]), "code rows"),
+    ]
+    for (w, keep), off, why in cases:
+        assert h.status_of("sq_grouped_fwd", ctypes.byref(w), off, vp(A16), vp(A16), None) == -1, why
+        assert why.split("[")[0].split("=")[0] in h.last_error(), (why, h.last_error())
+    w, keep = _gw()
+    assert h.status_of("sq_grouped_fwd", ctypes.byref(w), None, vp(A16), vp(A16), None) == -1
+    assert h.status_of("sq_grouped_fwd", ctypes.byref(w), _off([0, 0, 0, 0]), None, None, None) == 0
+    assert h.status_of("sq_grouped_bwd_dx", ctypes.byref(w), good_off, vp(A16 + 2), vp(A16), None) == -1
+    assert h.status_of("sq_grouped_scale_grad", ctypes.byref(w), good_off, vp(A16), vp(A16), None, None,
+                       None) == -1                                           # g is NULL
+    assert h.status_of("sq_grouped_project_lowrank", ctypes.byref(w), 0, 1.0, vp(A16), vp(A16), vp(A16), None,
+                       None, None, None) == -1                               # r = 0
+    assert h.status_of("sq_grouped_lowrank_grad", 0, 8, 8, 4, 1.0, vp(A16), vp(A16), vp(A16), vp(A16), vp(A16),
+                       None) == -1                                           # E = 0
+
+
+def test_variant_validation(built):
+    """The scale-family variants reject bad shapes, scales and groupings before any
+    device work; the control's empty batch is a no-op."""
+    h = pkg.Handle()
+    vp = ctypes.c_void_p
+    L = pkg._lib
+    assert h.status_of("sq_fit_scale_delta", 0, 8, 48, 1.0, vp(A16), None, vp(A16), vp(A16), None, None, None,
+                       None) == -1                                           # K % 32
+    assert h.status_of("sq_fit_scale_delta", 0, 8, 64, float("nan"), vp(A16), None, vp(A16), vp(A16), None, None,
+                       None, None) == -1                                     # ws2
+    assert h.status_of("sq_group_reduce", 8, 6, 4, vp(A16), vp(A16), None) == -1        # 4 does not divide 6
+    assert h.status_of("sq_group_reduce", 8, 6, 0, vp(A16), vp(A16), None) == -1
+    assert h.status_of("sq_project_group_delta", 1, 8, 6, 2, 0.5, vp(A16), vp(A16), vp(A16), None, None, None,
+                       None) == -1                                           # MXFP4 ws2
+    bad_n = L._SqControlWeight(12, 64, A16, A16)
+    assert h.status_of("sq_control_fwd", ctypes.byref(bad_n), vp(A16), 4, vp(A16), None) == -1
+    bad_w = L._SqControlWeight(8, 64, A16 + 2, A16)
+    assert h.status_of("sq_control_bwd_dx", ctypes.byref(bad_w), vp(A16), 4, vp(A16), None) == -1
+    ok = L._SqControlWeight(8, 64, A16, A16)
+    assert h.status_of("sq_control_fwd", ctypes.byref(ok), None, 0, None, None) == 0
+    assert h.status_of("sq_lowrank_product", 8, 8, 300, 1.0, vp(A16), vp(A16), vp(A16), None) == -1   # r > 256
