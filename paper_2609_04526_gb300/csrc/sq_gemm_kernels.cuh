@@ -453,11 +453,10 @@ __device__ __forceinline__ uint32_t load_unit_scale(const KParams &p, const uint
 
 // ------------------------------------------------------------- scale-gradient kernel
 //
-// D[n, k] = sum_m dY[m, n] X[m, k] on one CTA per SM: both operands are MN-major
-// TMA tiles (dY^T as two 64(n) x 64(m) boxes, X as four 64(k) x 64(m) boxes),
-// contraction over the tokens. The epilogue multiplies each dW element by its
-// E2M1 code and sums every block of B columns, applies the STE mask and writes
-// g[n, b]; the dW tile never leaves the SM.
+// D[n, k] = sum_m dY[m, n] X[m, k], contraction over the tokens: both operands
+// are MN-major TMA tiles (64 features x kSgradBK tokens per box). The epilogue
+// multiplies each dW element by its E2M1 code and sums every block of B columns,
+// applies the STE mask and writes g[n, b]; the dW tile never leaves the SM.
 
 // ------------------------------------------------------------- CTA-pair kernels
 //
@@ -603,6 +602,7 @@ struct PairCfg {
 };
 static_assert(PairCfg::kSmemBytes <= 232448, "pair kernel exceeds the opt-in shared memory of one CTA");
 static_assert(PairCfg::kMTile == 2 * PairCfg::kTile, "a pair tile is two halves");
+static_assert(PairCfg::kAStages == 2 * PairCfg::kStages, "half 1's activation slots are released with the decoded slots");
 static_assert(PairCfg::kEpiWarps == 8, "the epilogue maps warp w to lane quadrant w % 4 and column half w / 4");
 
 // Decode unit u (0..511) of this CTA's half at stage kb covers 32 consecutive
@@ -633,10 +633,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
   uint64_t *afull = bars;             // [SA] leader: both CTAs' activation tiles landed (1 arrival + 2 x kA tx)
-  uint64_t *aempty = afull + SA;      // [SA] pair MMAs reading activation slot a done   (multicast commit)
-  uint64_t *empty = aempty + SA;      // [S] pair MMAs reading decoded slot s done       (multicast commit)
+  uint64_t *aempty = afull + SA;      // [SA] pair MMAs reading half 0's slot a done     (multicast commit)
+  uint64_t *empty = aempty + SA;      // [S] pair MMAs of k-step s done: decoded slot s and
+                                      //     half 1's activation slot free      (multicast commit)
   uint64_t *pready = empty + S;       // [S] leader: both weight halves decoded          (1 arrival + st.async tx)
-  uint64_t *gready = pready + S;      // [S] leader: pready and half 0's afull seen by the gate (1 arrival)
+  uint64_t *gready = pready + S;      // [S] leader: pready and both halves' afull seen by the gate (1 arrival)
   uint64_t *cfull = gready + S;       // [SC] this CTA's code tile landed                 (1 arrival + tx)
   uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes      (kDecWarps arrivals)
   uint64_t *tfull = cempty + SC;      // [2] accumulator h of the tile complete          (multicast commit)
@@ -717,7 +718,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           for (int h = 0; h < 2; ++h, ++ja) {
             const int a = ja % SA;
             const uint32_t use = static_cast<uint32_t>(ja / SA);
-            if (ja >= SA && !(ok = mbar_wait(&aempty[a], (use & 1u) ^ 1u, abort_flag, p.err))) break;
+            // half 0's slot is freed by the commit after its 8 MMAs; half 1's together
+            // with the decoded slot, by the commit that ends k-step ja / 2 - S
+            if (ja >= SA && !(ok = h == 0 ? mbar_wait(&aempty[a], (use & 1u) ^ 1u, abort_flag, p.err)
+                                          : mbar_wait(&empty[(ja / 2) % S],
+                                                      (static_cast<uint32_t>(ja / 2 / S) & 1u) ^ 1u, abort_flag, p.err)))
+              break;
             if (rank == 0) mbar_arrive_expect_tx(&afull[a], C::kATx);
             const uint32_t bar = mapa_shared(smem_u32(&afull[a]), 0);
             // two 128 x 64 boxes (one per 64-wide K chunk, 16 KiB apart)
@@ -791,11 +797,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
-    // A k-step needs both decoded weight halves and the activation tile of half 0,
-    // which the gate warp folds into one barrier (gready), and, 8 MMAs later, the
-    // activation tile of half 1 (loaded last, so it gets those 1024 cycles of
-    // slack). Every barrier wait of this thread costs issue time the tensor core
-    // cannot hide, so it spins on the barriers (test_wait) and polls none between MMAs.
+    // A k-step needs both decoded weight halves and the activation tiles of both
+    // halves, which the gate warp folds into one barrier (gready). Every barrier
+    // wait and every commit of this thread costs issue time the tensor core cannot
+    // hide, so it waits once per k-step, spinning (test_wait), polls nothing between
+    // MMAs and commits twice: half 0's activation slot after its 8 MMAs (the TMA
+    // warp refills it a half step early) and, after all 16, the decoded slot together
+    // with half 1's activation slot.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
       // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
@@ -819,8 +827,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
                 !(ok = mbar_spin_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
               break;
             if (kb == 0) tc_fence_after();
-            if (h == 1 && !(ok = mbar_spin(&afull[a], static_cast<uint32_t>((2 * it + 1) / SA) & 1u, abort_flag, p.err)))
-              break;
             const uint32_t d_tmem = tmem_base + h * kTmemCols;
             const uint64_t a0 = ad_base + static_cast<uint64_t>(a * (C::kA >> 4));
 #pragma unroll
@@ -829,7 +835,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
               const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
               umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
             }
-            umma_commit_pair_mc(&aempty[a]);
+            if (h == 0) umma_commit_pair_mc(&aempty[a]);
             if (kb == num_k - 1) umma_commit_pair_mc(&tfull[h]);  // the epilogue may start on accumulator h
             if (++a == SA) a = 0;
           }
@@ -848,7 +854,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ gate (leader CTA)
     // Waits, for each k-step, for both decoded halves (pready, a cluster-scope
     // acquire that costs a few hundred cycles even on a completed barrier) and for
-    // the activation tile of half 0 (afull), then hands the step to the MMA thread
+    // the activation tiles of both halves (afull), then hands the step to the MMA thread
     // through one CTA-local barrier. It also arms pready with the signal
     // bytes of each use (decode warps may signal before it is armed: the missing
     // arrival keeps the phase open).
@@ -859,6 +865,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         const int s = it % S;
         if (!mbar_spin_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
         if (!mbar_spin(&afull[(2 * it) % SA], static_cast<uint32_t>((2 * it) / SA) & 1u, abort_flag, p.err)) break;
+        if (!mbar_spin(&afull[(2 * it + 1) % SA], static_cast<uint32_t>((2 * it + 1) / SA) & 1u, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
@@ -1139,8 +1146,8 @@ struct SgradPairCfg {
   static constexpr int kTmaWarp = 4;
   static constexpr int kMmaWarp = 5;
   static constexpr int kThreads = 192;
-  static constexpr int kBK = kSgradBK;         // tokens per stage: 4 MMAs of K = 16
-  static constexpr int kStages = 6;
+  static constexpr int kBK = kSgradBK;         // tokens per stage: 8 MMAs of K = 16
+  static constexpr int kStages = 3;
   static constexpr int kA = 128 * kBK * 2;     // 16 KiB: this CTA's 128 n-rows of dY^T, two MN atoms of 64 n
   static constexpr int kB = 128 * kBK * 2;     // 16 KiB: this CTA's 128 k-columns of X, two MN atoms of 64 k
   static constexpr int kAtom = kBK * 128;      // bytes of one 64-wide MN atom (kBK rows of 128 B)

@@ -17,7 +17,7 @@ enum GemmMode : int {
 // Rows of one activation TMA box of the pair kernels (the rows a CTA holds of a tile half).
 constexpr int kBM = 128;
 // Tokens per shared-memory stage of the scale-gradient kernel (also the height of its TMA boxes).
-constexpr int kSgradBK = 64;
+constexpr int kSgradBK = 128;
 
 struct GemmArgs {
   int mode;

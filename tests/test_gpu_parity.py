@@ -145,6 +145,42 @@ def test_layer_step_and_merge_c5(h):
     assert 0.005 < frac < 0.2, frac
 
 
+@pytest.mark.parametrize("key,fmt,M,N,K", [SMALL[0], SMALL[2]], ids=["c1", "mx_ragged"])
+def test_merged_artifact_is_the_trained_weight(h, key, fmt, M, N, K):
+    """max|dW| = 0 in weight space (Sec. 3, merge): the artifact (unchanged codes plus the
+    merged scale plane) decodes to exactly the weight the training forward used (codes plus
+    the projected bytes), and the kernels give bit-identical Y, dX and g on both."""
+    from paper_2609_04526_gb300 import synth
+    import paper_2609_04526_gb300 as pkg
+    wl = _wl(key, fmt, M, N, K)
+    lin = wl.linears[0]
+    w = synth.gen_weight(wl, lin, device="cuda")
+    X = synth.gen_act(wl, lin.x, device="cuda")
+    dY = synth.gen_dy(wl, lin, device="cuda")
+    L = synth.gen_latent(wl, lin, w, device="cuda")
+    L[::3] *= 2                      # a step of one binade on every third row, so E8M0 bytes move too
+    codes0 = w.codes.clone()
+    q, mask = h.sq_project_scales(wl.fmt, L, w.ws2)
+    art = w.scales.clone()
+    h.sq_merge(wl.fmt, L, w.ws2, art)
+    h.sq_sync()
+    c = host(w.codes)
+    W_train = oracle.decode_weight(fmt, c, host(q), w.ws2, N, K)
+    W_art = oracle.decode_weight(fmt, c, host(art), w.ws2, N, K)
+    assert np.isfinite(W_train).all()
+    assert np.max(np.abs(W_art - W_train)) == 0.0
+    assert not np.array_equal(host(art), host(w.scales))       # the merge did move bytes
+    outs = []
+    for s in (q, art):
+        qw = pkg.QuantWeight(wl.fmt, N, K, w.codes, s, w.ws2)
+        outs.append((h.sq_fwd(qw, X), h.sq_bwd_dx(qw, dY), h.sq_scale_grad(qw, X, dY, mask=mask)))
+    h.sq_sync()
+    for a, b in zip(*outs):
+        assert torch.equal(a.view(torch.int16) if a.dtype == torch.bfloat16 else a.view(torch.int32),
+                           b.view(torch.int16) if b.dtype == torch.bfloat16 else b.view(torch.int32))
+    assert torch.equal(w.codes, codes0)
+
+
 def _edge_latents(fmt, ws2):
     rng = np.random.default_rng(99)
     vals = []
