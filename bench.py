@@ -64,7 +64,7 @@ def parse_args():
 
 def profiled_traffic(workload):
     """DRAM bytes per launch measured by ncu for each kernel kind (profiles/); a kind
-    is left out when the source file of its kernel changed since the capture."""
+    is left out when a source file of its kernel changed since the capture."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"traffic_{workload}_layer_step.json")
     if not os.path.exists(path):
@@ -73,8 +73,13 @@ def profiled_traffic(workload):
         prof = json.load(f)
     out = {}
     for kind, entry in prof.get("kernels", {}).items():
-        src = os.path.join(ROOT, "paper_2609_04526_gb300", "csrc", entry.get("source", ""))
-        if os.path.isfile(src) and hashlib.sha256(open(src, "rb").read()).hexdigest() == entry.get("source_sha256"):
+        srcs = [os.path.join(ROOT, "paper_2609_04526_gb300", "csrc", f) for f in entry.get("sources", [])]
+        if not srcs or not all(os.path.isfile(f) for f in srcs):
+            continue
+        h = hashlib.sha256()
+        for f in srcs:
+            h.update(open(f, "rb").read())
+        if h.hexdigest() == entry.get("sources_sha256"):
             out[kind] = entry
     return out
 
@@ -715,7 +720,7 @@ def run_ours(args):
                          "traffic": traffic.get(dom, {}).get("dram_bytes_per_launch"),
                          "algorithmic_bytes": traffic.get(dom, {}).get("algorithmic_bytes_per_launch"),
                          "traffic_note": "ncu dram bytes per launch, mean over the layer's 7 launches of this kernel "
-                                         "(profiles/traffic_c5_layer_step.json); null if its source changed since",
+                                         "(profiles/traffic_c5_layer_step.json); null if its sources changed since",
                          "peak_source": f"{pk['source']} bf16 sustained"},
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels,
