@@ -93,6 +93,14 @@ const char *sq_last_error(sq_handle h);
  * Returns SQ_OK, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
 sq_status sq_sync(sq_handle h, void *stream);
 
+/* Self-test of the failure path: launches one thread that waits on a shared-
+ * memory barrier nothing arrives on, with the bounded wait every contraction
+ * kernel uses (1 s); when it runs out the thread records the timeout in the
+ * device error word and returns, so the context stays usable. The next sq_sync
+ * on `stream` returns SQ_ERR_DEVICE_TIMEOUT (and clears the word). Returns
+ * SQ_OK once enqueued, SQ_ERR_UNSUPPORTED / SQ_ERR_CUDA as the compute calls. */
+sq_status sq_selftest_wait_timeout(sq_handle h, void *stream);
+
 /* Forward, Sec. 3 "Scale-QLoRA forward": Y[m,n] = sum_k X[m,k] W[n,k].
  * X  device bf16 [M, K] (input), Y device bf16 [M, N] (output, overwritten).
  * Accumulation in fp32; ws2 is applied to the fp32 accumulator; Y is rounded

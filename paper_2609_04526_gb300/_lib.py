@@ -30,7 +30,8 @@ EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_s
            "sq_rollback", "sq_swap_scales", "sq_count_diff", "sq_scale_grad_noalloc", "sq_grouped_fwd",
            "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
            "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad", "sq_fit_scale_delta", "sq_group_reduce",
-           "sq_project_group_delta", "sq_control_fwd", "sq_control_bwd_dx", "sq_control_grad", "sq_lowrank_product")
+           "sq_project_group_delta", "sq_control_fwd", "sq_control_bwd_dx", "sq_control_grad", "sq_lowrank_product",
+           "sq_selftest_wait_timeout")
 
 
 class SQError(RuntimeError):
@@ -74,6 +75,7 @@ def load() -> ctypes.CDLL:
     L.sq_last_error.argtypes = [vp]
     L.sq_last_error.restype = ctypes.c_char_p
     L.sq_sync.argtypes = [vp, vp]
+    L.sq_selftest_wait_timeout.argtypes = [vp, vp]
     L.sq_fwd.argtypes = [vp, W, vp, i64, vp, vp]
     L.sq_bwd_dx.argtypes = [vp, W, vp, i64, vp, vp]
     L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
@@ -201,6 +203,11 @@ class Handle:
     # entry points ------------------------------------------------------------
     def sq_sync(self, stream=None):
         self._check(self._L.sq_sync(self._h, _stream(stream)))
+
+    def sq_selftest_wait_timeout(self, stream=None):
+        """Enqueue a bounded wait that runs out (about 1 s); the next sq_sync raises
+        SQError with status SQ_ERR_DEVICE_TIMEOUT."""
+        self._check(self._L.sq_selftest_wait_timeout(self._h, _stream(stream)))
 
     def sq_fwd(self, w: QuantWeight, X: torch.Tensor, Y: Optional[torch.Tensor] = None, stream=None):
         M = X.shape[0]

@@ -559,6 +559,17 @@ sq_status sq_sync(sq_handle h, void *stream) {
   SQ_GUARD_END
 }
 
+sq_status sq_selftest_wait_timeout(sq_handle h, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const cudaError_t e = sqi::launch_wait_probe(dev->err_word, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "launching the wait self-test");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
 sq_status sq_fwd(sq_handle h, const sq_weight *w, const uint16_t *X, int64_t M, uint16_t *Y, void *stream) {
   if (!h) return SQ_ERR_INVALID_ARG;
   SQ_GUARD_BEGIN

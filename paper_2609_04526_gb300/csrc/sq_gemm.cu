@@ -26,4 +26,21 @@ cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtenso
   return launch_sgrad<1, false>(p, tmA, tmB, sm_count, stream);
 }
 
+// The failure-path self-test: the same bounded spin the contraction kernels use,
+// on a barrier whose phase never completes.
+__global__ void sq_wait_probe_kernel(int *err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  abort_flag = 0;
+  fence_barrier_init();
+  (void)mbar_spin(&bar, 0u, &abort_flag, err);  // runs out after kWaitLimitNs and records it
+}
+
+cudaError_t launch_wait_probe(int *err, cudaStream_t stream) {
+  sq_wait_probe_kernel<<<1, 32, 0, stream>>>(err);
+  return cudaGetLastError();
+}
+
 }  // namespace sqi

@@ -90,6 +90,9 @@ cudaError_t launch_lowrank_product(int64_t N, int64_t G, int r, float alpha_over
 // 32-row x 32-column boxes, 64-byte swizzle; null for MODE_SGRAD).
 cudaError_t launch_gemm(const GemmArgs &a, const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap *tmOut,
                         int sm_count, cudaStream_t stream);
+// One thread waiting on a barrier nothing arrives on, bounded like every kernel wait:
+// records kErrWaitTimeout in *err and returns (the failure-path self-test).
+cudaError_t launch_wait_probe(int *err, cudaStream_t stream);
 
 // Projection / merge of `count` latents. With ws2_per (device, one float per
 // expert; NVFP4 only) the latents are the planes of several experts, `plane` (a

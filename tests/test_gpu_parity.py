@@ -260,6 +260,30 @@ def test_empty_batch_and_sync(h):
     assert (g == 0).all()
 
 
+def test_bounded_wait_runs_out_and_the_context_survives(h):
+    """The failure path without a fault: a wait on a barrier nothing arrives on runs
+    out after its bound, the next sync reports SQ_ERR_DEVICE_TIMEOUT, the sync after
+    it is clean, and the same handle and context still compute correct results."""
+    import time
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import synth
+    h.sq_sync()
+    t0 = time.time()
+    h.sq_selftest_wait_timeout()
+    with pytest.raises(pkg.SQError) as info:
+        h.sq_sync()
+    waited = time.time() - t0
+    assert info.value.status == -5 and "bounded device wait" in str(info.value)
+    assert 0.5 < waited < 30, waited
+    h.sq_sync()                                   # the error word was cleared
+    wl = synth.custom("t", NV, 70, 136, 2080, seed=3)
+    w, X, dY = setup_linear(wl, wl.linears[0])
+    Y = h.sq_fwd(w, X)
+    h.sq_sync()
+    ref = oracle.fwd(NV, host(w.codes), host(w.scales), w.ws2, hbits(X))
+    assert_close(f64(Y), ref, what="Y after a device timeout")
+
+
 def test_invalid_args_on_device(h):
     import paper_2609_04526_gb300 as pkg
     from paper_2609_04526_gb300 import synth
