@@ -251,7 +251,7 @@ def run_step(h, S, stream, events=None, ins=None):
         mark()
 
 
-LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge kernels
+LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge (+1 where the scale gradient splits its tokens)
 LAUNCHES_PER_LINEAR_LOWRANK = 8  # + the adapter gradients' three kernels (dB, dA partials, dA reduce)
 
 
@@ -725,7 +725,8 @@ def run_ours(args):
             "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
             "kernels": kernels,
             "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": (LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl * args.steps,
+            "gpu_launches": ((LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl
+                             + sum(h.sq_scale_grad_workspace(st["qw"], S.wl.M)[0] > 1 for st in S.lin)) * args.steps,
             "clocks": clk,
         }
         line.update(context)

@@ -121,9 +121,22 @@ sq_status sq_bwd_dx(sq_handle h, const sq_weight *w, const uint16_t *dY, int64_t
  * X device bf16 [M, K], dY device bf16 [M, N], mask device u8 [N, K/B] or NULL,
  * g device fp32 [N, K/B] (output, overwritten; all zero when M == 0). The
  * weight's scale bytes are not read (w->scales may be NULL).
- * The dW = dY^T X tile is reduced per block on chip and never written. */
+ * The dW = dY^T X tile is reduced per block on chip and never written.
+ * A weight with few 256 x 256 tiles (fewer than a handful of waves over the
+ * GPU's SMs) has its M tokens cut into up to 8 parts: each part's unmasked
+ * partial gradient goes to scratch the handle owns, and a second kernel adds
+ * the parts in order and applies the mask (deterministic; the fp32 sums round
+ * differently from an unsplit launch). The scratch is allocated, or grown, on
+ * the first call that needs it (cudaMalloc, which may synchronise the device);
+ * sq_scale_grad_workspace reports the split and the scratch size. */
 sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
                         const uint8_t *mask, float *g, void *stream);
+
+/* The token split sq_scale_grad uses for this weight shape and M on the current
+ * device: *splits (host, nullable) = the number of parts (1 = a single launch, no
+ * scratch), *bytes (host, nullable) = the handle scratch it needs, splits * N * (K/B)
+ * * 4 (0 when unsplit). Host-only; returns SQ_ERR_INVALID_ARG for a bad shape. */
+sq_status sq_scale_grad_workspace(sq_handle h, const sq_weight *w, int64_t M, int32_t *splits, int64_t *bytes);
 
 /* Grid projection, Sec. 3 QAST round_grid with the ceiling clamp of the
  * stability recipe (ii)/(iii), for count = N*G latent scales (absolute units):

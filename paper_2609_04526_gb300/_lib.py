@@ -31,7 +31,7 @@ EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_s
            "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
            "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad", "sq_fit_scale_delta", "sq_group_reduce",
            "sq_project_group_delta", "sq_control_fwd", "sq_control_bwd_dx", "sq_control_grad", "sq_lowrank_product",
-           "sq_selftest_wait_timeout")
+           "sq_selftest_wait_timeout", "sq_scale_grad_workspace")
 
 
 class SQError(RuntimeError):
@@ -76,6 +76,7 @@ def load() -> ctypes.CDLL:
     L.sq_last_error.restype = ctypes.c_char_p
     L.sq_sync.argtypes = [vp, vp]
     L.sq_selftest_wait_timeout.argtypes = [vp, vp]
+    L.sq_scale_grad_workspace.argtypes = [vp, W, i64, vp, vp]
     L.sq_fwd.argtypes = [vp, W, vp, i64, vp, vp]
     L.sq_bwd_dx.argtypes = [vp, W, vp, i64, vp, vp]
     L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
@@ -224,6 +225,15 @@ class Handle:
         wc = w._c()
         self._check(self._L.sq_bwd_dx(self._h, ctypes.byref(wc), _ptr(dY), M, _ptr(dX), _stream(stream)))
         return dX
+
+    def sq_scale_grad_workspace(self, w: QuantWeight, M: int):
+        """(splits, scratch bytes) of sq_scale_grad for this weight shape and M tokens."""
+        sp = ctypes.c_int32(0)
+        nb = ctypes.c_int64(0)
+        wc = w._c()
+        self._check(self._L.sq_scale_grad_workspace(self._h, ctypes.byref(wc), int(M), ctypes.byref(sp),
+                                                    ctypes.byref(nb)))
+        return sp.value, nb.value
 
     def sq_scale_grad(self, w: QuantWeight, X: torch.Tensor, dY: torch.Tensor, mask: Optional[torch.Tensor] = None,
                       g: Optional[torch.Tensor] = None, stream=None):

@@ -39,6 +39,8 @@ struct DeviceState {
   size_t workspace_bytes;
   TableSlot tables[kTableSlots];
   int next_table;
+  float *partial = nullptr;  // token-split partial planes of the dense scale gradient, grown on demand
+  size_t partial_bytes = 0;
 };
 
 constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
@@ -185,6 +187,25 @@ sq_status check_buf(sq_handle h, const void *p, const char *name) {
     return fail(h, SQ_ERR_CUDA, "internal error (host exception)");              \
   }
 
+// Token splits of a dense scale gradient of M tokens on this device (sgrad_splits).
+int sgrad_splits_of(const DeviceState *dev, const sq_weight *w, int64_t M) {
+  const int64_t tiles = ((w->N + sqi::kSgradTile - 1) / sqi::kSgradTile) * ((w->K + sqi::kSgradTile - 1) / sqi::kSgradTile);
+  return sqi::sgrad_splits(tiles, dev->sm_count / 2, M);
+}
+
+// The split partial planes on the current device, at least `bytes` (a larger buffer
+// replaces the old one; cudaFree waits for the work that may still use it).
+sq_status ensure_partial(sq_handle h, DeviceState *dev, size_t bytes) {
+  if (bytes <= dev->partial_bytes) return SQ_OK;
+  cudaError_t e;
+  if (dev->partial && (e = cudaFree(dev->partial)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(partial planes)");
+  dev->partial = nullptr;
+  dev->partial_bytes = 0;
+  if ((e = cudaMalloc(&dev->partial, bytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(partial planes)");
+  dev->partial_bytes = bytes;
+  return SQ_OK;
+}
+
 sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr, const void *b_ptr, int64_t M,
                    void *out, const uint8_t *mask, cudaStream_t stream) {
   DeviceState *dev = nullptr;
@@ -222,6 +243,14 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
   a.out = out;
   a.mask = mask;
   a.err = dev->err_word;
+  if (mode == sqi::MODE_SGRAD) {
+    a.splits = sgrad_splits_of(dev, w, M);
+    if (a.splits > 1) {
+      const size_t bytes = static_cast<size_t>(a.splits) * w->N * (w->K / block_of(w->fmt)) * sizeof(float);
+      SQ_TRY(ensure_partial(h, dev, bytes));
+      a.partial = dev->partial;
+    }
+  }
   cudaError_t e = sqi::launch_gemm(a, tmA, tmB, mode == sqi::MODE_SGRAD ? nullptr : &tmOut, dev->sm_count, stream);
   if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
   return SQ_OK;
@@ -509,6 +538,7 @@ sq_status sq_destroy(sq_handle h) {
     if (cudaSetDevice(d.device) == cudaSuccess) {
       cudaFree(d.err_word);
       if (d.workspace) cudaFree(d.workspace);
+      if (d.partial) cudaFree(d.partial);
       for (auto &t : d.tables) {
         if (t.done) {
           cudaEventSynchronize(t.done);
@@ -591,6 +621,21 @@ sq_status sq_bwd_dx(sq_handle h, const sq_weight *w, const uint16_t *dY, int64_t
   SQ_TRY(check_buf(h, dY, "dY"));
   SQ_TRY(check_buf(h, dX, "dX"));
   return run_gemm(h, sqi::MODE_DX, w, dY, nullptr, M, dX, nullptr, static_cast<cudaStream_t>(stream));
+  SQ_GUARD_END
+}
+
+sq_status sq_scale_grad_workspace(sq_handle h, const sq_weight *w, int64_t M, int32_t *splits, int64_t *bytes) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  SQ_TRY(check_weight(h, w, false));
+  SQ_TRY(check_tokens(h, M));
+  if (!splits && !bytes) return fail(h, SQ_ERR_INVALID_ARG, "splits and bytes are both NULL");
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  const int s = M == 0 ? 1 : sgrad_splits_of(dev, w, M);
+  if (splits) *splits = s;
+  if (bytes) *bytes = s > 1 ? static_cast<int64_t>(s) * w->N * (w->K / block_of(w->fmt)) * 4 : 0;
+  return SQ_OK;
   SQ_GUARD_END
 }
 

@@ -20,7 +20,9 @@
 //
 // SGRAD (sq_sgrad_pair_kernel): a cluster of two CTAs per 256 x 256 tile of
 // dW = dY^T X with both operands as MN-major TMA tiles; each CTA's epilogue
-// reduces code x dW per block for its 128 rows.
+// reduces code x dW per block for its 128 rows. A dense launch with few tiles
+// may cut the tokens into parts (KParams::splits): each (part, tile) unit writes
+// a partial plane, which sq_split_reduce_kernel (sq_gemm.cu) adds in order.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs): on expiry the CTA records
 // kErrWaitTimeout in the device error word, stops issuing, drains what it has
@@ -370,6 +372,8 @@ struct KParams {
   int total;             // tiles of the launch
   const uint8_t *gtab;   // grouped: the device expert table (GroupMaps[E], tile_start, rows, ws2); else null
   int groups;            // experts of a grouped launch, 1 for a dense one
+  int splits = 1;            // dense scale gradient: token splits (total = tiles x splits units)
+  float *partial = nullptr;  // ... with splits > 1: [splits, N, G] partial planes (no mask)
 };
 
 // Tuning constants of the decode warps (compile-time; the defaults are the measured best).
@@ -1184,11 +1188,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
   const int cluster = blockIdx.x >> 1;
   const int nclusters = gridDim.x >> 1;
   const int total = p.total;
-  // token stages of a tile: all M tokens, or the expert's own M_e in a grouped
-  // launch (an expert without tokens gets zero gradient blocks)
-  auto stages_of = [&](int e) -> int {
-    const int64_t m = GR ? static_cast<int64_t>(group_rows(p, e)) : p.M;
-    return static_cast<int>((m + C::kBK - 1) / C::kBK);
+  // Unit u of the launch: tile (tm, tn) (of expert e in a grouped launch) over the
+  // token stages [m0, m0 + kBK * num_k): all M tokens, the expert's own M_e, or in
+  // a dense launch cut into token splits, part sp of them (an expert or part
+  // without tokens gets zero gradient blocks). Returns num_k.
+  const int tiles_per_split = p.tiles_m * p.tiles_n;
+  const int64_t split_tokens =
+      ((p.M + p.splits - 1) / p.splits + C::kBK - 1) / C::kBK * C::kBK;  // a multiple of kBK
+  auto unit_of = [&](int u, int &e, int &tm, int &tn, int &sp, int32_t &m0) -> int {
+    if (GR) {
+      resolve_tile<GR, kSgradGroup>(p, u, e, tm, tn);
+      sp = 0;
+      m0 = 0;
+      return static_cast<int>((static_cast<int64_t>(group_rows(p, e)) + C::kBK - 1) / C::kBK);
+    }
+    sp = p.splits > 1 ? u / tiles_per_split : 0;
+    resolve_tile<GR, kSgradGroup>(p, u - sp * tiles_per_split, e, tm, tn);
+    const int64_t first = static_cast<int64_t>(sp) * split_tokens;
+    const int64_t len = p.M - first < split_tokens ? p.M - first : split_tokens;
+    m0 = static_cast<int32_t>(first);
+    return len > 0 ? static_cast<int>((len + C::kBK - 1) / C::kBK) : 0;
   };
 
   auto stage_a = [&](int s) { return smem + s * C::kStageBytes; };
@@ -1225,9 +1244,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
       int e = 0, e_seen = -1;
       const CUtensorMap *mA = &tmA, *mB = &tmB;
       for (int tile = cluster; tile < total && ok; tile += nclusters) {
-        int tm, tn;
-        resolve_tile<GR, kSgradGroup>(p, tile, e, tm, tn);
-        const int num_k = stages_of(e);
+        int tm, tn, sp;
+        int32_t m0;
+        const int num_k = unit_of(tile, e, tm, tn, sp, m0);
         if (GR && e != e_seen && num_k > 0) {  // the expert's own token rows of dY and X (an expert
           mA = &group_maps(p, e)->m[0];        // without tokens has no descriptors and loads nothing)
           mB = &group_maps(p, e)->m[1];
@@ -1243,7 +1262,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
           if (it >= S && !(ok = mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.err))) break;
           if (rank == 0) mbar_arrive_expect_tx(&full[s], C::kTx);
           const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
-          const int32_t kc = kb * C::kBK;
+          const int32_t kc = m0 + kb * C::kBK;
           for (int j = 0; j < 2; ++j) tma_load_2d_pair(smem_u32(stage_a(s)) + j * C::kAtom, mA, bar, row0 + 64 * j, kc);
           for (int j = 0; j < 2; ++j) tma_load_2d_pair(smem_u32(stage_b(s)) + j * C::kAtom, mB, bar, col0 + 64 * j, kc);
         }
@@ -1265,9 +1284,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
       bool ok = true;
       int e = 0;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
-        int tm, tn;
-        resolve_tile<GR, kSgradGroup>(p, tile, e, tm, tn);
-        const int num_k = stages_of(e);
+        int tm, tn, sp;
+        int32_t m0;
+        const int num_k = unit_of(tile, e, tm, tn, sp, m0);
         const int ab = tc & 1;
         const uint32_t au = static_cast<uint32_t>(tc >> 1);
         if (tc >= 2 && !(ok = mbar_spin_cluster(&tempty[ab], (au & 1u) ^ 1u, abort_flag, p.err))) break;
@@ -1302,13 +1321,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
     int tc = 0;
     int e = 0;
     for (int tile = cluster; tile < total; tile += nclusters, ++tc) {
-      int tm, tn;
-      resolve_tile<GR, kSgradGroup>(p, tile, e, tm, tn);
-      // the expert's code plane (the multiplicative control: its bf16 weights), gradient plane and mask
+      int tm, tn, sp;
+      int32_t m0;
+      const int num_k = unit_of(tile, e, tm, tn, sp, m0);
+      // the expert's code plane (the multiplicative control: its bf16 weights), gradient plane and
+      // mask; a token split writes its own partial plane, masked when the parts are added
       const uint8_t *codes = GR ? p.codes + e * p.N * (p.K / 2) : p.codes;
-      float *g = static_cast<float *>(p.out) + (GR ? e * p.N * G : 0);
-      const uint8_t *mask = p.mask ? p.mask + (GR ? e * p.N * G : 0) : nullptr;
-      const bool empty_sum = GR && stages_of(e) == 0;  // no tokens: the accumulator was never written
+      float *g = p.splits > 1 ? p.partial + sp * p.N * G : static_cast<float *>(p.out) + (GR ? e * p.N * G : 0);
+      const uint8_t *mask = p.mask && p.splits == 1 ? p.mask + (GR ? e * p.N * G : 0) : nullptr;
+      const bool empty_sum = num_k == 0;  // no tokens: the accumulator was never written
       const int64_t n = static_cast<int64_t>(tm) * C::kTile + 128 * rank + r;
       const int64_t col0 = static_cast<int64_t>(tn) * C::kTile;
       const int ab = tc & 1;

@@ -29,6 +29,8 @@ struct GemmArgs {
   void *out;             // Y [M,N] bf16 | dX [M,K] bf16 | g [N,K/B] f32
   const uint8_t *mask;   // [N, K/B] or null (MODE_SGRAD only)
   int *err;              // device error word
+  int splits = 1;            // MODE_SGRAD: token splits (sgrad_splits)
+  float *partial = nullptr;  // MODE_SGRAD with splits > 1: [splits, N, K/B] fp32 partial sums
 };
 
 // Expert table of a grouped launch, built by the host for each call and copied
@@ -53,6 +55,30 @@ __host__ __device__ constexpr size_t group_table_bytes(int E) { return group_off
 constexpr int kPairMTile = 512;
 constexpr int kPairNTile = 256;
 constexpr int kSgradTile = 256;
+
+// Token splits of a dense scale-gradient launch. Each 256 x 256 tile contracts over
+// all M tokens, so a launch with few tiles (q/k/v/o of the layer: 256 or 64) leaves
+// much of its last wave idle. The tokens are then cut into up to kMaxSgradSplits
+// parts of at least kMinSplitTokens each, one unit per (part, tile); every part
+// writes a partial gradient plane and a second kernel adds the parts in order.
+// Cost model, in units of one full-M tile on one cluster: ceil(tiles * s /
+// clusters) / s, plus 1 % per extra part (the partial planes' traffic).
+constexpr int kMaxSgradSplits = 8;
+constexpr int64_t kMinSplitTokens = 2048;
+inline int sgrad_splits(int64_t tiles, int clusters, int64_t M) {
+  if (tiles <= 0 || clusters <= 0) return 1;
+  int best = 1;
+  double best_cost = static_cast<double>((tiles + clusters - 1) / clusters);
+  for (int s = 2; s <= kMaxSgradSplits; ++s) {
+    if (M < s * kMinSplitTokens) break;
+    const double cost = static_cast<double>((tiles * s + clusters - 1) / clusters) / s + 0.01 * (s - 1);
+    if (cost < best_cost - 1e-9) {
+      best = s;
+      best_cost = cost;
+    }
+  }
+  return best;
+}
 
 struct GroupedArgs {
   int mode;

@@ -88,6 +88,18 @@ def test_buffer_and_token_validation(built):
     assert h.status_of("sq_merge", 0, 4, 16, 1.0, vp(A16), vp(A16), vp(A16 + 4), None, None) == -1
 
 
+def test_scale_grad_workspace_validation(built):
+    """The split query validates the weight, the token count and its outputs before
+    it looks at a device."""
+    h = pkg.Handle()
+    vp = ctypes.c_void_p
+    sp, nb = ctypes.c_int32(0), ctypes.c_int64(0)
+    assert h.status_of("sq_scale_grad_workspace", ctypes.byref(_w(N=12)), 4096, ctypes.byref(sp), ctypes.byref(nb)) == -1
+    assert h.status_of("sq_scale_grad_workspace", ctypes.byref(_w()), -1, ctypes.byref(sp), ctypes.byref(nb)) == -1
+    assert h.status_of("sq_scale_grad_workspace", ctypes.byref(_w()), 4096, None, None) == -1
+    assert h.status_of("sq_scale_grad_workspace", None, 4096, ctypes.byref(sp), None) == -1
+
+
 def test_empty_batch_is_a_noop_without_device(built):
     """M == 0 for the forward / input gradient enqueues nothing."""
     h = pkg.Handle()

@@ -181,6 +181,36 @@ def test_merged_artifact_is_the_trained_weight(h, key, fmt, M, N, K):
     assert torch.equal(w.codes, codes0)
 
 
+@pytest.mark.parametrize("fmt,M,N,K", [(NV, 9000, 1024, 512), (MX, 8320, 520, 1024)], ids=["nv", "mx"])
+def test_token_split_scale_gradient(h, fmt, M, N, K):
+    """A weight with few scale-gradient tiles (8 and 12 here) cuts its tokens into
+    parts, the last one ragged: the masked sum of the parts matches the oracle on
+    every block of sampled rows, the query reports the split and its scratch, two
+    runs give identical bits, and the unsplit launch on the first 2048 tokens (a
+    single part) matches too."""
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom(f"split{fmt}", fmt, M, N, K, seed=11 + fmt, kind="outlier" if fmt else "gauss")
+    w, X, dY = setup_linear(wl, wl.linears[0])
+    G = K // (16 if fmt == NV else 32)
+    splits, nbytes = h.sq_scale_grad_workspace(w, M)
+    assert splits == 4 and nbytes == splits * N * G * 4
+    assert h.sq_scale_grad_workspace(w, 2048) == (1, 0)
+    rng = np.random.default_rng(M)
+    mask = torch.from_numpy(rng.integers(0, 2, size=(N, G), dtype=np.uint8)).cuda()
+    g1 = h.sq_scale_grad(w, X, dY, mask=mask)
+    g2 = h.sq_scale_grad(w, X, dY, mask=mask)
+    g0 = h.sq_scale_grad(w, X[:2048], dY[:2048])
+    h.sq_sync()
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    rows = np.unique(np.concatenate([[0, 255, 256, N - 1], rng.integers(0, N, 20)]))
+    codes = host(w.codes)
+    ref = oracle.scale_grad(fmt, codes, hbits(X), hbits(dY), mask=host(mask), rows=rows)
+    full = oracle.scale_grad(fmt, codes, hbits(X), hbits(dY), rows=rows)
+    assert_close(f64(g1)[rows], ref, rms=float(np.sqrt(np.mean(full ** 2))), what="split g*mask")
+    ref0 = oracle.scale_grad(fmt, codes, hbits(X[:2048]), hbits(dY[:2048]), rows=rows)
+    assert_close(f64(g0)[rows], ref0, what="unsplit g")
+
+
 def _edge_latents(fmt, ws2):
     rng = np.random.default_rng(99)
     vals = []
