@@ -34,7 +34,10 @@
  *    is an empty batch). Every device pointer must be 16-byte aligned.
  *  - Argument errors return SQ_ERR_INVALID_ARG before anything is launched; the
  *    text is in sq_last_error(h). No exception or abort crosses the ABI.
- *  - A handle is not thread-safe; use one handle per host thread.
+ *  - A handle is not thread-safe; use one handle per host thread. The scratch a
+ *    handle owns (a split scale gradient's partial planes; the adapter kernels'
+ *    partial sums) is one buffer per kind and device: calls of one handle that
+ *    use it must run on one stream or be ordered by the caller.
  *  - Device waits are bounded: a wait that runs out sets a device error word
  *    instead of hanging; sq_sync reports it as SQ_ERR_DEVICE_TIMEOUT.
  *  - Decoded weights are formed exactly in bf16 (the code x scale-byte product
