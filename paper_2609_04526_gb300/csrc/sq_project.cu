@@ -400,13 +400,38 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
       for (int c = 0; c < 4; ++c) acc[q][c] = fmaf(bv[q], av[c], acc[q][c]);
   }
   uint32_t nan_count = 0;
+  // four consecutive blocks of a row per thread: one 4-byte load of the base bytes and
+  // one 4-byte (16-byte for the latent) store per output where the row allows it
+  const bool vec = (G & 3) == 0;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
+    const int64_t n = n0 + ty * 4 + q, bq = b0 + tx * 4;
+    if (n >= N) continue;
+    const int64_t i0 = n * G + bq;
+    if (vec && bq + 3 < G) {
+      const uint32_t base4 = __ldg(reinterpret_cast<const uint32_t *>(base + i0));
+      uint32_t by4 = 0, mk4 = 0;
+      float Lv[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float L = fmaf(aor, acc[q][c], scale_value<FMT>((base4 >> (8 * c)) & 0xFFu, ws2));
+        uint32_t by, mk, na;
+        project_one<FMT>(L, ws2, cap, by, mk, na);
+        by4 |= by << (8 * c);
+        mk4 |= mk << (8 * c);
+        nan_count += na;
+        Lv[c] = L;
+      }
+      *reinterpret_cast<uint32_t *>(bytes_out + i0) = by4;
+      if (mask_out) *reinterpret_cast<uint32_t *>(mask_out + i0) = mk4;
+      if (latent_out) *reinterpret_cast<float4 *>(latent_out + i0) = make_float4(Lv[0], Lv[1], Lv[2], Lv[3]);
+      continue;
+    }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      const int64_t n = n0 + ty * 4 + q, b = b0 + tx * 4 + c;
-      if (n < N && b < G) {
-        const int64_t i = n * G + b;
+      const int64_t b = bq + c;
+      if (b < G) {
+        const int64_t i = i0 + c;
         const float L = fmaf(aor, acc[q][c], scale_value<FMT>(base[i], ws2));
         uint32_t by, mk, na;
         project_one<FMT>(L, ws2, cap, by, mk, na);

@@ -64,6 +64,8 @@ CASES = [
     ("lr_mx", MX, 300, 96, 64),
     ("lr_rmax", NV, 37, 16, 256),
     ("lr_mx_ragged", MX, 65, 144, 33),
+    ("lr_nv_g6", NV, 24, 6, 5),        # G % 4 != 0: the per-block store path
+    ("lr_mx_g71", MX, 72, 71, 9),
 ]
 
 
