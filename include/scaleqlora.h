@@ -131,7 +131,10 @@ sq_status sq_bwd_dx(sq_handle h, const sq_weight *w, const uint16_t *dY, int64_t
  * the parts in order and applies the mask (deterministic; the fp32 sums round
  * differently from an unsplit launch). The scratch is allocated, or grown, on
  * the first call that needs it (cudaMalloc, which may synchronise the device);
- * sq_scale_grad_workspace reports the split and the scratch size. */
+ * sq_scale_grad_workspace reports the split and the scratch size. A call that
+ * would have to grow the scratch while `stream` is being captured into a CUDA
+ * graph returns SQ_ERR_UNSUPPORTED instead: size it with one call outside the
+ * capture, after which captured calls allocate nothing. */
 sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, const uint16_t *dY, int64_t M,
                         const uint8_t *mask, float *g, void *stream);
 

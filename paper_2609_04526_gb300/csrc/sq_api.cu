@@ -194,10 +194,17 @@ int sgrad_splits_of(const DeviceState *dev, const sq_weight *w, int64_t M) {
 }
 
 // The split partial planes on the current device, at least `bytes` (a larger buffer
-// replaces the old one; cudaFree waits for the work that may still use it).
-sq_status ensure_partial(sq_handle h, DeviceState *dev, size_t bytes) {
+// replaces the old one; cudaFree waits for the work that may still use it). Growing
+// it is refused while `stream` is being captured into a graph (no allocation there).
+sq_status ensure_partial(sq_handle h, DeviceState *dev, size_t bytes, cudaStream_t stream) {
   if (bytes <= dev->partial_bytes) return SQ_OK;
-  cudaError_t e;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(stream, &cap);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
+  if (cap != cudaStreamCaptureStatusNone)
+    return fail(h, SQ_ERR_UNSUPPORTED,
+                "the scale gradient needs %zu bytes of scratch: make one call outside graph capture first "
+                "(sq_scale_grad_workspace reports the size)", bytes);
   if (dev->partial && (e = cudaFree(dev->partial)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(partial planes)");
   dev->partial = nullptr;
   dev->partial_bytes = 0;
@@ -247,7 +254,7 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
     a.splits = sgrad_splits_of(dev, w, M);
     if (a.splits > 1) {
       const size_t bytes = static_cast<size_t>(a.splits) * w->N * (w->K / block_of(w->fmt)) * sizeof(float);
-      SQ_TRY(ensure_partial(h, dev, bytes));
+      SQ_TRY(ensure_partial(h, dev, bytes, stream));
       a.partial = dev->partial;
     }
   }

@@ -211,6 +211,36 @@ def test_token_split_scale_gradient(h, fmt, M, N, K):
     assert_close(f64(g0)[rows], ref0, what="unsplit g")
 
 
+def test_split_scale_gradient_in_a_cuda_graph():
+    """A fresh handle refuses to grow its split scratch inside graph capture (nothing
+    is enqueued); after one call outside capture, the captured split scale gradient
+    replays to the same bits as the direct call."""
+    import paper_2609_04526_gb300 as pkg
+    from paper_2609_04526_gb300 import synth
+    wl = synth.custom("graph", NV, 9000, 1024, 512, seed=5)
+    w, X, dY = setup_linear(wl, wl.linears[0])
+    h2 = pkg.Handle()
+    assert h2.sq_scale_grad_workspace(w, 9000)[0] > 1
+    s = torch.cuda.Stream()
+    g = torch.zeros(1024, 32, device="cuda")
+    graph = torch.cuda.CUDAGraph()
+    with pytest.raises(pkg.SQError) as ei:
+        with torch.cuda.graph(graph, stream=s):
+            h2.sq_scale_grad(w, X, dY, g=g, stream=s)
+    assert ei.value.status == -2 and "outside graph capture" in str(ei.value)
+    ref = h2.sq_scale_grad(w, X, dY, stream=s)      # sizes the scratch
+    h2.sq_sync(s)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        h2.sq_scale_grad(w, X, dY, g=g, stream=s)
+    g.zero_()
+    torch.cuda.synchronize()
+    graph.replay()
+    torch.cuda.synchronize()
+    h2.sq_sync(s)
+    assert torch.equal(g.view(torch.int32), ref.view(torch.int32))
+
+
 def _edge_latents(fmt, ws2):
     rng = np.random.default_rng(99)
     vals = []
