@@ -37,7 +37,11 @@
  *  - A handle is not thread-safe; use one handle per host thread. The scratch a
  *    handle owns (a split scale gradient's partial planes; the adapter kernels'
  *    partial sums) is one buffer per kind and device: calls of one handle that
- *    use it must run on one stream or be ordered by the caller.
+ *    use it must run on one stream or be ordered by the caller. It is allocated,
+ *    or grown, by the first call that needs it; a call that would grow it while
+ *    its stream is being captured into a CUDA graph returns SQ_ERR_UNSUPPORTED,
+ *    so make one call outside the capture first. Grouped calls that take an
+ *    sq_grouped_weight copy a host-built expert table and cannot be captured.
  *  - Device waits are bounded: a wait that runs out sets a device error word
  *    instead of hanging; sq_sync reports it as SQ_ERR_DEVICE_TIMEOUT.
  *  - Decoded weights are formed exactly in bf16 (the code x scale-byte product

@@ -669,10 +669,16 @@ sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, cons
 }
 
 // The handle's scratch on the current device, at least `bytes` (a larger buffer
-// replaces the old one; cudaFree waits for the work that may still use it).
-static sq_status ensure_workspace(sq_handle h, DeviceState *dev, size_t bytes) {
+// replaces the old one; cudaFree waits for the work that may still use it). Growing
+// it is refused while `stream` is being captured into a graph (no allocation there).
+static sq_status ensure_workspace(sq_handle h, DeviceState *dev, size_t bytes, cudaStream_t stream) {
   if (bytes <= dev->workspace_bytes) return SQ_OK;
-  cudaError_t e;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(stream, &cap);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
+  if (cap != cudaStreamCaptureStatusNone)
+    return fail(h, SQ_ERR_UNSUPPORTED,
+                "the adapter kernels need %zu bytes of scratch: make one call outside graph capture first", bytes);
   if (dev->workspace && (e = cudaFree(dev->workspace)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(workspace)");
   dev->workspace = nullptr;
   dev->workspace_bytes = 0;
@@ -845,7 +851,7 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
   SQ_TRY(check_buf(h, g, "g"));
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
-  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count)));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count), st));
   e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
                                dev->sm_count, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");
@@ -987,7 +993,8 @@ sq_status sq_lowrank_product(sq_handle h, int64_t N, int64_t G, int32_t r, float
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
   SQ_TRY(check_buf(h, out, "out"));
-  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_product_workspace(N, G, r, dev->sm_count)));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_product_workspace(N, G, r, dev->sm_count),
+                          static_cast<cudaStream_t>(stream)));
   cudaError_t e = sqi::launch_lowrank_product(N, G, r, alpha_over_r, B, A, out, static_cast<float *>(dev->workspace),
                                               dev->sm_count, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(h, e, "low-rank product launch");
@@ -1126,7 +1133,7 @@ sq_status sq_grouped_lowrank_grad(sq_handle h, int32_t E, int64_t N, int64_t G, 
   SQ_TRY(check_buf(h, g, "g"));
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
-  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count, E)));
+  SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count, E), st));
   e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
                                dev->sm_count, st, E);
   if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter gradient launch");
