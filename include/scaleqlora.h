@@ -239,7 +239,9 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
  * allocates nothing: the kernel's scratch (the device error word its bounded
  * waits set) lives in a file-scope static __device__ array of 256 bytes that
  * every GPU loading the library holds until the process exits.
- *  - Arguments, layouts and results are those of sq_scale_grad.
+ *  - Arguments, layouts and results are those of sq_scale_grad, always in one
+ *    pass over the tokens: where sq_scale_grad cuts them into parts (its
+ *    partial planes need scratch), the two results agree up to fp32 rounding.
  *  - Scratch limit: 256 bytes; this kernel needs one 4-byte word for any M, N, K,
  *    and a call whose need exceeded the array would return SQ_ERR_INVALID_ARG.
  *  - The first call on each device sets up (checks the device, looks up the
