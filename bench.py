@@ -252,7 +252,7 @@ def run_step(h, S, stream, events=None, ins=None):
 
 
 LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge (+1 where the scale gradient splits its tokens)
-LAUNCHES_PER_LINEAR_LOWRANK = 8  # + the adapter gradients' three kernels (dB, dA partials, dA reduce)
+LAUNCHES_PER_LINEAR_LOWRANK = 9  # + the adapter gradients' four kernels (dB and dA products, each chunk sum)
 
 
 def kernel_work(S):
