@@ -1080,6 +1080,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         tc_fence_after();
         const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * quad;
         const uint32_t t_buf = t_row + h * kTmemCols;
+        // input gradient and grouped launches: the last 32-column group is read into
+        // registers and stored after the accumulator is released
+        constexpr bool kHold = MODE == MODE_DX || GR;
+        uint32_t held[16];
 #pragma unroll 1
         for (int j = 0; j < C::kTile / 2; j += 32) {
           const int c = cbase + j;
@@ -1092,6 +1096,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
             const __nv_bfloat162 h2 =
                 __floats2bfloat162_rn(__uint_as_float(v[2 * q]) * scale, __uint_as_float(v[2 * q + 1]) * scale);
             packed[q] = *reinterpret_cast<const uint32_t *>(&h2);
+          }
+          if (kHold && j == C::kTile / 2 - 32) {
+#pragma unroll
+            for (int q = 0; q < 16; ++q) held[q] = packed[q];
+            break;
           }
           if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
           __syncwarp();
@@ -1119,6 +1128,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           } else {
             st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
                             mapa_shared(smem_u32(&tempty[h]), 0));
+          }
+        }
+        if (kHold) {  // the held group: staged and stored now
+          const int c = cbase + C::kTile / 2 - 32;
+          if (lane == 0) bulk_wait_read<0>();
+          __syncwarp();
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), held[4 * q], held[4 * q + 1], held[4 * q + 2],
+                         held[4 * q + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
+            bulk_commit_group();
           }
         }
       }
