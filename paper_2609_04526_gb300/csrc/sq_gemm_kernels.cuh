@@ -1051,7 +1051,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // 32 (w % 4) .. +31 and columns 128 (w / 4) .. +127, 32 columns at a time:
     // it scales and rounds them to bf16 into a 32 x 32 box in shared memory
     // (64-byte swizzle) and stores the box with TMA, which writes whole row
-    // segments and clips the ragged edges of the output.
+    // segments and clips the ragged edges of the output. The input-gradient and
+    // grouped kernels keep a warp's last group in registers and release the
+    // accumulator before staging it (measured: it helps those, not the forward).
     const int quad = warp & 3;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
     const int cbase = (warp >> 2) * (C::kTile / 2);
