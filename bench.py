@@ -36,6 +36,9 @@ METRIC = "fwd+dX+dScale TFLOP/s per layer & fraction of GB300 bf16 tensor peak"
 UNIT = "TFLOP/s"
 KINDS = ("project", "fwd", "dx", "sgrad", "merge")
 KINDS_LOWRANK = ("project", "fwd", "dx", "sgrad", "adapter_grad", "merge")
+# GB300 datasheet figures (dense, no sparsity): the fractions against these sit beside
+# the ones against the measured torch matmul / copy rates.
+DATASHEET = {"bf16_tflops": 2250.0, "hbm_gbs": 7900.0}
 ADAPTER_RANK = 58  # the paper's Llama-3-8B scale rank (Sec. 5 recipe)
 
 
@@ -96,30 +99,112 @@ def peaks():
 
 # --------------------------------------------------------------------- clocks
 
+class _Nvml:
+    """Read-only NVML queries through ctypes (libnvidia-ml ships with the driver):
+    SM clock, its maximum, power draw and the active clock-event reasons."""
+    SM = 1  # NVML_CLOCK_SM
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+               0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, uuid):
+        import ctypes
+        self.c = ctypes
+        self.lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if self.lib.nvmlInit_v2() != 0:
+            raise RuntimeError("nvmlInit failed")
+        self.dev = ctypes.c_void_p()
+        if self.lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(self.dev)) != 0:
+            raise RuntimeError("no NVML device for " + uuid)
+        try:
+            self.reasons_fn = self.lib.nvmlDeviceGetCurrentClocksEventReasons
+        except AttributeError:
+            self.reasons_fn = self.lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        v = ctypes.c_uint()
+        self.max_mhz = float(v.value) if self.lib.nvmlDeviceGetMaxClockInfo(self.dev, self.SM, ctypes.byref(v)) == 0 \
+            else None
+
+    def sample(self):
+        c = self.c
+        mhz, mw, reasons = c.c_uint(), c.c_uint(), c.c_ulonglong()
+        if self.lib.nvmlDeviceGetClockInfo(self.dev, self.SM, c.byref(mhz)) != 0:
+            return None
+        self.lib.nvmlDeviceGetPowerUsage(self.dev, c.byref(mw))
+        self.reasons_fn(self.dev, c.byref(reasons))
+        return float(mhz.value), mw.value / 1000.0, int(reasons.value)
+
+    def close(self):
+        self.lib.nvmlShutdown()
+
+
 class ClockSampler:
-    """nvidia-smi samples (200 ms) of SM clock and throttle reasons during the timed region."""
+    """SM clock, power and throttle reasons sampled every 25 ms during the timed
+    region (NVML through ctypes; nvidia-smi at 50 ms where NVML is unavailable)."""
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
+    PERIOD_S = 0.025
 
     def __init__(self, device_index):
         self.proc = None
-        self.path = None
-        exe = shutil.which("nvidia-smi")
-        if not exe:
-            return
+        self.thread = None
+        self.samples = []
+        self.source = None
         try:
             uuid = "GPU-" + str(torch.cuda.get_device_properties(device_index).uuid)
         except Exception:
             uuid = None
+        if uuid:
+            try:
+                self.nvml = _Nvml(uuid)
+                self._start_thread()
+                self.source = "nvml 25 ms"
+                return
+            except Exception:
+                self.nvml = None
+        exe = shutil.which("nvidia-smi")
+        if not exe:
+            return
         fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
         os.close(fd)
         cmd = [exe] + (["-i", uuid] if uuid else []) + ["--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
-                                                         "-lms", "200"]
+                                                         "-lms", "50"]
         self.fh = open(self.path, "w")
         self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+        self.source = "nvidia-smi 50 ms"
+
+    def _start_thread(self):
+        import threading
+        self.stop_evt = threading.Event()
+
+        def loop():
+            while not self.stop_evt.is_set():
+                v = self.nvml.sample()
+                if v is not None:
+                    self.samples.append(v)
+                self.stop_evt.wait(self.PERIOD_S)
+
+        self.thread = threading.Thread(target=loop, daemon=True)
+        self.thread.start()
+
+    def _summary(self, sm, smax, watts, reasons):
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "sm_min_mhz": min(sm),
+                "power_w_median": statistics.median(watts) if watts else None, "reasons": sorted(reasons),
+                "samples": len(sm), "source": self.source}
 
     def stop(self):
+        if self.thread is not None:
+            self.stop_evt.set()
+            self.thread.join(timeout=5)
+            self.nvml.close()
+            reasons = set()
+            for _, _, r in self.samples:
+                for bit, name in _Nvml.REASONS.items():
+                    if r & bit:
+                        reasons.add(name)
+            return self._summary([m for m, _, _ in self.samples], self.nvml.max_mhz,
+                                 [w for _, w, _ in self.samples], reasons)
         if not self.proc:
             return None
         self.proc.terminate()
@@ -128,7 +213,7 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.fh.close()
-        sm, smax, reasons = [], [], set()
+        sm, smax, watts, reasons = [], [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
         with open(self.path) as f:
             for line in f:
@@ -138,16 +223,26 @@ class ClockSampler:
                 try:
                     sm.append(float(parts[0]))
                     smax.append(float(parts[1]))
+                    watts.append(float(parts[2]))
                 except ValueError:
                     continue
                 for name, v in zip(names, parts[4:8]):
                     if v.lower().startswith("active"):
                         reasons.add(name)
         os.unlink(self.path)
-        if not sm:
-            return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return self._summary(sm, max(smax) if smax else None, watts, reasons)
+
+
+def per_ghz(kernels, clk):
+    """Clock-normalised figures of each kernel kind: throughput per GHz of the median
+    sampled SM clock, and the step's share of that kind in millions of SM cycles."""
+    if not clk or not clk.get("sm_mhz"):
+        return
+    ghz = clk["sm_mhz"] / 1e3
+    for k in kernels.values():
+        k["per_ghz"] = k["achieved"] / ghz
+        k["per_ghz_unit"] = k["unit"] + " per GHz"
+        k["mcycles_per_step"] = k["ms_per_step"] * clk["sm_mhz"] / 1e3
 
 
 # --------------------------------------------------------------------- workload
@@ -168,6 +263,7 @@ class LayerState:
             G = lin.K // wl.block
             st = dict(
                 lin=lin, base_scales=w.scales, ws2=w.ws2, codes=w.codes, latent=L,
+                codes0=w.codes.clone(),                     # the frozen code plane, to verify it is untouched
                 art=w.scales.clone(),                       # artifact scale plane rewritten by the merge
                 qbytes=torch.empty_like(w.scales),          # projected (on-grid) scale bytes used by the forward
                 mask=torch.empty_like(w.scales),
@@ -277,6 +373,42 @@ def kernel_work(S):
 
 # --------------------------------------------------------------------- oracle sample
 
+def snapshot_outputs(S, n_y, n_dx, n_rows, seed=0):
+    """A seeded sample of the last timed step's outputs, read back right after the
+    timed region (before any other leg reuses the buffers): Y and dX elements, full
+    rows of the masked scale gradient, the projected bytes, STE mask and merged
+    artifact planes, the NaN and changed-byte counters, and whether every code plane
+    still equals the copy taken before the first step."""
+    rng = np.random.default_rng(seed)
+    out = {}
+    for st in S.lin:
+        l = st["lin"]
+        M = S.wl.M
+        ms, ns = rng.integers(0, M, n_y), rng.integers(0, l.N, n_y)
+        ms2, ks = rng.integers(0, M, n_dx), rng.integers(0, l.K, n_dx)
+        rows = rng.integers(0, l.N, n_rows)
+        dev = st["Y"].device
+
+        def ti(a):
+            return torch.from_numpy(a).to(dev)
+
+        out[l.name] = dict(
+            ms=ms, ns=ns, ms2=ms2, ks=ks, rows=rows,
+            Y=st["Y"][ti(ms), ti(ns)].double().cpu().numpy(), dX=st["dX"][ti(ms2), ti(ks)].double().cpu().numpy(),
+            g=st["g"][ti(rows)].double().cpu().numpy(), qbytes=st["qbytes"].cpu().numpy(),
+            mask=st["mask"].cpu().numpy(), art=st["art"].cpu().numpy(), nonfinite=int(st["nonfinite"].item()),
+            changed=int(st["changed"].item()), codes_unchanged=bool(torch.equal(st["codes"], st["codes0"])))
+    return out
+
+
+def _err_over_bound(gpu, ref, rms):
+    """Worst |gpu - ref| / (2e-2 |ref| + 1e-3 rms) over a sample (<= 1 passes), and the count above 1."""
+    bound = 2e-2 * np.abs(ref) + 1e-3 * rms
+    r = np.abs(gpu - ref) / np.maximum(bound, 1e-300)
+    r = np.where(np.isnan(r), np.inf, r)
+    return float(r.max()) if r.size else 0.0, int((r > 1).sum())
+
+
 def oracle_sample(wl, host, linears, n_y, n_dx, n_rows, n_plane, seed=0):
     """Time the float64 oracle on a bounded sample of one step and extrapolate
     the full step's CPU time from each part's per-unit rate."""
@@ -310,6 +442,73 @@ def oracle_sample(wl, host, linears, n_y, n_dx, n_rows, n_plane, seed=0):
     return t_full, t_spent, (f"{n_y} Y and {n_dx} dX elements, {n_rows} full scale-gradient rows and "
                              f"{n_plane} latents through projection and merge, per linear ({', '.join(desc)}); "
                              "full-step time extrapolated from each part's measured per-element rate")
+
+
+def oracle_check_sample(wl, host, linears, n_plane, snap):
+    """The CPU baseline: time the float64 oracle on the sampled outputs of one step
+    and extrapolate the full step's CPU time from each part's per-unit rate; the
+    same sample checks the last timed step. The oracle projects each latent plane
+    itself (untimed), and its own bytes and mask feed its contractions: the GPU's
+    projected bytes, mask, merged plane and counters must equal the oracle's bit for
+    bit, Y, dX and g rows agree within 2e-2 relative + 1e-3 x RMS, and the code
+    planes must be unchanged."""
+    import oracle
+    t_full = 0.0
+    t_spent = 0.0
+    desc = []
+    ver = {"ok": True, "linears": 0, "y_elements": 0, "dx_elements": 0, "g_rows": 0, "plane_bytes_bit_exact": 0,
+           "code_planes_unchanged": True, "worst_err_over_bound": {"Y": 0.0, "dX": 0.0, "g": 0.0}, "failures": []}
+    for lin in linears:
+        d = host[lin.name]
+        v = snap[lin.name]
+        M, N, K = wl.M, lin.N, lin.K
+        rb, rm, rnf = oracle.project(wl.fmt, d["latent"], d["ws2"])
+        # the artifact plane before the last step held the previous step's merge, the same projection
+        rs, _, rch = oracle.merge(wl.fmt, d["latent"], rb, d["ws2"], want_delta=False)
+        planes = [("bytes", v["qbytes"], rb), ("mask", v["mask"], rm), ("merged", v["art"], rs)]
+        for what, a, b in planes:
+            if np.array_equal(a, b):
+                ver["plane_bytes_bit_exact"] += a.size
+            else:
+                ver["failures"].append(f"{lin.name}: {what} plane differs in {int((a != b).sum())} bytes")
+        if v["nonfinite"] != rnf or v["changed"] != rch:
+            ver["failures"].append(f"{lin.name}: counters {v['nonfinite']}/{v['changed']} vs oracle {rnf}/{rch}")
+        if not v["codes_unchanged"]:
+            ver["code_planes_unchanged"] = False
+            ver["failures"].append(f"{lin.name}: code plane changed")
+        t0 = time.perf_counter()
+        Yr = oracle.fwd_at(wl.fmt, d["codes"], rb, d["ws2"], d["X"], v["ms"], v["ns"])
+        t1 = time.perf_counter()
+        dXr = oracle.dx_at(wl.fmt, d["codes"], rb, d["ws2"], d["dY"], v["ms2"], v["ks"])
+        t2 = time.perf_counter()
+        gr = oracle.scale_grad(wl.fmt, d["codes"], d["X"], d["dY"], mask=rm, rows=v["rows"])
+        t3 = time.perf_counter()
+        Lp = d["latent"].reshape(-1)[:n_plane]
+        oracle.project(wl.fmt, Lp, d["ws2"])
+        t4 = time.perf_counter()
+        oracle.merge(wl.fmt, Lp, d["scales"].reshape(-1)[:n_plane], d["ws2"], want_delta=False)
+        t5 = time.perf_counter()
+        for what, a, b in (("Y", v["Y"], Yr), ("dX", v["dX"], dXr), ("g", v["g"], gr)):
+            worst, bad = _err_over_bound(a, b, float(np.sqrt(np.mean(b ** 2))))
+            ver["worst_err_over_bound"][what] = max(ver["worst_err_over_bound"][what], worst)
+            if bad:
+                ver["failures"].append(f"{lin.name}: {bad} {what} values outside the tolerance")
+        ver["linears"] += 1
+        ver["y_elements"] += len(Yr)
+        ver["dx_elements"] += len(dXr)
+        ver["g_rows"] += len(v["rows"])
+        blocks = N * (K // wl.block)
+        n_y, n_dx, n_rows = len(v["ms"]), len(v["ks"]), len(v["rows"])
+        t_full += ((t1 - t0) * (M * N / n_y) + (t2 - t1) * (M * K / n_dx) + (t3 - t2) * (N / n_rows)
+                   + (t4 - t3 + t5 - t4) * (blocks / min(n_plane, blocks)))
+        t_spent += t5 - t0
+        desc.append(lin.name)
+    ver["ok"] = not ver["failures"]
+    n0 = snap[linears[0].name]
+    return t_full, t_spent, (f"{len(n0['ms'])} Y and {len(n0['ks'])} dX elements, {len(n0['rows'])} full "
+                             f"scale-gradient rows and {n_plane} latents through projection and merge, per linear "
+                             f"({', '.join(desc)}); full-step time extrapolated from each part's measured per-element "
+                             "rate"), ver
 
 
 def host_copies(S, linears):
@@ -610,6 +809,13 @@ def run_ours(args):
     h.sq_sync(stream)
     ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
     ms_step = ms_total / args.steps
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    n_threads = None
+    if want_cpu:
+        import oracle
+        oracle.lib()
+        n_threads = oracle.num_threads()
+        snap = snapshot_outputs(S, n_y=1024, n_dx=1024, n_rows=6 * n_threads, seed=12345)
 
     kind_ms = {k: 0.0 for k in kinds}
     kind_launch = {k: 0 for k in kinds}
@@ -630,6 +836,10 @@ def run_ours(args):
         else:
             ach = by[kind] / t / 1e9
             kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
+    for kind, k in kernels.items():
+        k["frac_vs_datasheet"] = k["achieved"] / (DATASHEET["bf16_tflops"] if k["unit"] == "TFLOP/s"
+                                                  else DATASHEET["hbm_gbs"])
+    per_ghz(kernels, clk)
     dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
     traffic = {} if args.lowrank else profiled_traffic(wl.key)  # the profile is of the default step's kernels
     for kind in kinds:
@@ -694,13 +904,11 @@ def run_ours(args):
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
-        oracle.lib()
+    verified = None
+    if want_cpu:
         host = host_copies(S, list(wl.linears))
-        t_full, t_spent, desc = oracle_sample(wl, host, list(wl.linears), n_y=1024, n_dx=1024,
-                                              n_rows=6 * oracle.num_threads(), n_plane=1 << 18)
-        cpu = {"value": flops_step / t_full / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+        t_full, t_spent, desc, verified = oracle_check_sample(wl, host, list(wl.linears), n_plane=1 << 18, snap=snap)
+        cpu = {"value": flops_step / t_full / 1e12, "unit": UNIT, "cores": n_threads, "kind": "oracle",
                "sample": desc, "sample_seconds": round(t_spent, 2), "extrapolated_step_seconds": round(t_full, 1)}
 
     if rank == 0:
@@ -721,8 +929,14 @@ def run_ours(args):
                          "algorithmic_bytes": traffic.get(dom, {}).get("algorithmic_bytes_per_launch"),
                          "traffic_note": "ncu dram bytes per launch, mean over the layer's 7 launches of this kernel "
                                          "(profiles/traffic_c5_layer_step.json); null if its sources changed since",
-                         "peak_source": f"{pk['source']} bf16 sustained"},
-            "fraction_of_peak": {"bf16_burst": value / world / pk["bf16"], "bf16_sustained": value / world / pk["bf16_sustained"]},
+                         "peak_source": f"{pk['source']} bf16 sustained (torch.matmul 8192^3 held for 4 s)",
+                         "frac_vs_datasheet": k["achieved"] / DATASHEET["bf16_tflops"]},
+            "fraction_of_peak": {"bf16_burst_measured_matmul": value / world / pk["bf16"],
+                                 "bf16_sustained_measured_matmul": value / world / pk["bf16_sustained"],
+                                 "bf16_datasheet_dense": value / world / DATASHEET["bf16_tflops"]},
+            "per_ghz": ({"value": value / world / (clk["sm_mhz"] / 1e3), "unit": "TFLOP/s per GHz (median SM clock)"}
+                        if clk and clk.get("sm_mhz") else None),
+            "verified": verified,
             "kernels": kernels,
             "e2e": e2e, "cpu_baseline": cpu,
             "gpu_launches": ((LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl
@@ -957,6 +1171,10 @@ def run_moe(args):
         else:
             ach = by[kind] / t / 1e9
             kernels[kind] = {"ms_per_step": t * 1e3, "achieved": ach, "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
+    for k in kernels.values():
+        k["frac_vs_datasheet"] = k["achieved"] / (DATASHEET["bf16_tflops"] if k["unit"] == "TFLOP/s"
+                                                  else DATASHEET["hbm_gbs"])
+    per_ghz(kernels, clk)
     dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
     value = wl.flops() * args.steps * world / (ms_total / 1e3) / 1e12
 

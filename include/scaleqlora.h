@@ -40,8 +40,12 @@
  *    use it must run on one stream or be ordered by the caller. It is allocated,
  *    or grown, by the first call that needs it; a call that would grow it while
  *    its stream is being captured into a CUDA graph returns SQ_ERR_UNSUPPORTED,
- *    so make one call outside the capture first. Grouped calls that take an
- *    sq_grouped_weight copy a host-built expert table and cannot be captured.
+ *    so make one call outside the capture first. A buffer that a capture has
+ *    used is never freed while the handle lives: when a later call grows it,
+ *    the old buffer is kept (and freed by sq_destroy), so graphs captured
+ *    earlier replay correctly until the handle is destroyed. Grouped calls that
+ *    take an sq_grouped_weight copy a host-built expert table and cannot be
+ *    captured.
  *  - Device waits are bounded: a wait that runs out sets a device error word
  *    instead of hanging; sq_sync reports it as SQ_ERR_DEVICE_TIMEOUT.
  *  - Decoded weights are formed exactly in bf16 (the code x scale-byte product
@@ -244,9 +248,11 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
  *    partial planes need scratch), the two results agree up to fp32 rounding.
  *  - Scratch limit: 256 bytes; this kernel needs one 4-byte word for any M, N, K,
  *    and a call whose need exceeded the array would return SQ_ERR_INVALID_ARG.
- *  - The first call on each device sets up (checks the device, looks up the
- *    array's device address with cudaGetSymbolAddress); make that first call
- *    before any stream capture.
+ *  - The first call on each device sets up (checks the device, resolves the
+ *    driver's tensor-map encoder); make that first call before any stream
+ *    capture. Every call, with the device current, looks up the array's device
+ *    address with cudaGetSymbolAddress (no allocation), so the address stays
+ *    right if the device's primary context is reset and the module reloaded.
  *  - Every call on a device shares the array: the error word is cleared at the
  *    start of each call, and calls that overlap on the GPU race on it.
  *  - device_status: device int32 or NULL; if given, it receives the error word

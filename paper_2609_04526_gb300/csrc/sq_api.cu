@@ -31,16 +31,24 @@ struct TableSlot {
 };
 constexpr int kTableSlots = 4;
 
+// Device scratch that grows on demand. Once a graph capture has recorded the buffer
+// it is never freed while the handle lives: growing it then retires the old buffer
+// (freed by sq_destroy), so graphs captured earlier keep valid pointers.
+struct Scratch {
+  void *ptr = nullptr;
+  size_t bytes = 0;
+  bool captured = false;        // a capture has recorded ptr
+  std::vector<void *> retired;  // earlier buffers recorded by captures
+};
+
 struct DeviceState {
   int device;
   int sm_count;
   int *err_word;         // device int, written by kernels whose bounded waits ran out
-  void *workspace;       // scratch of the adapter-gradient kernels, grown on demand
-  size_t workspace_bytes;
+  Scratch workspace;     // scratch of the adapter-gradient kernels
   TableSlot tables[kTableSlots];
   int next_table;
-  float *partial = nullptr;  // token-split partial planes of the dense scale gradient, grown on demand
-  size_t partial_bytes = 0;
+  Scratch partial;       // token-split partial planes of the dense scale gradient
 };
 
 constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
@@ -103,7 +111,12 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   int *err_word = nullptr;
   if ((e = cudaMalloc(&err_word, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(error word)");
   if ((e = cudaMemset(err_word, 0, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(error word)");
-  h->devices.push_back(DeviceState{dev, sms, err_word, nullptr, 0, {}, 0});
+  DeviceState d{};
+  d.device = dev;
+  d.sm_count = sms;
+  d.err_word = err_word;
+  d.next_table = 0;
+  h->devices.push_back(std::move(d));
   *out = &h->devices.back();
   return SQ_OK;
 }
@@ -193,24 +206,42 @@ int sgrad_splits_of(const DeviceState *dev, const sq_weight *w, int64_t M) {
   return sqi::sgrad_splits(tiles, dev->sm_count / 2, M);
 }
 
-// The split partial planes on the current device, at least `bytes` (a larger buffer
-// replaces the old one; cudaFree waits for the work that may still use it). Growing
-// it is refused while `stream` is being captured into a graph (no allocation there).
-sq_status ensure_partial(sq_handle h, DeviceState *dev, size_t bytes, cudaStream_t stream) {
-  if (bytes <= dev->partial_bytes) return SQ_OK;
+// Scratch `s` on the current device, at least `bytes`. Growing it is refused while
+// `stream` is being captured into a graph (no allocation there); a buffer that was
+// used during a capture is retired instead of freed when it grows. `need` names the
+// scratch in the error text.
+sq_status ensure_scratch(sq_handle h, Scratch &s, size_t bytes, cudaStream_t stream, const char *need) {
   cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
   cudaError_t e = cudaStreamIsCapturing(stream, &cap);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
-  if (cap != cudaStreamCaptureStatusNone)
-    return fail(h, SQ_ERR_UNSUPPORTED,
-                "the scale gradient needs %zu bytes of scratch: make one call outside graph capture first "
-                "(sq_scale_grad_workspace reports the size)", bytes);
-  if (dev->partial && (e = cudaFree(dev->partial)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(partial planes)");
-  dev->partial = nullptr;
-  dev->partial_bytes = 0;
-  if ((e = cudaMalloc(&dev->partial, bytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(partial planes)");
-  dev->partial_bytes = bytes;
+  const bool capturing = cap != cudaStreamCaptureStatusNone;
+  if (bytes <= s.bytes) {
+    if (capturing) s.captured = true;
+    return SQ_OK;
+  }
+  if (capturing)
+    return fail(h, SQ_ERR_UNSUPPORTED, "%s needs %zu bytes of scratch: make one call outside graph capture first", need,
+                bytes);
+  if (s.ptr) {
+    if (s.captured)
+      s.retired.push_back(s.ptr);
+    else if ((e = cudaFree(s.ptr)) != cudaSuccess)  // waits for the work that may still use it
+      return cuda_fail(h, e, "cudaFree(scratch)");
+  }
+  s.ptr = nullptr;
+  s.bytes = 0;
+  s.captured = false;
+  if ((e = cudaMalloc(&s.ptr, bytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(scratch)");
+  s.bytes = bytes;
   return SQ_OK;
+}
+
+void free_scratch(Scratch &s) {
+  if (s.ptr) cudaFree(s.ptr);
+  for (void *p : s.retired) cudaFree(p);
+  s.ptr = nullptr;
+  s.bytes = 0;
+  s.retired.clear();
 }
 
 sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr, const void *b_ptr, int64_t M,
@@ -254,8 +285,9 @@ sq_status run_gemm(sq_handle h, int mode, const sq_weight *w, const void *a_ptr,
     a.splits = sgrad_splits_of(dev, w, M);
     if (a.splits > 1) {
       const size_t bytes = static_cast<size_t>(a.splits) * w->N * (w->K / block_of(w->fmt)) * sizeof(float);
-      SQ_TRY(ensure_partial(h, dev, bytes, stream));
-      a.partial = dev->partial;
+      SQ_TRY(ensure_scratch(h, dev->partial, bytes, stream,
+                            "the split scale gradient (sq_scale_grad_workspace reports the size)"));
+      a.partial = static_cast<float *>(dev->partial.ptr);
     }
   }
   cudaError_t e = sqi::launch_gemm(a, tmA, tmB, mode == sqi::MODE_SGRAD ? nullptr : &tmOut, dev->sm_count, stream);
@@ -544,8 +576,8 @@ sq_status sq_destroy(sq_handle h) {
   for (auto &d : h->devices) {
     if (cudaSetDevice(d.device) == cudaSuccess) {
       cudaFree(d.err_word);
-      if (d.workspace) cudaFree(d.workspace);
-      if (d.partial) cudaFree(d.partial);
+      free_scratch(d.workspace);
+      free_scratch(d.partial);
       for (auto &t : d.tables) {
         if (t.done) {
           cudaEventSynchronize(t.done);
@@ -668,23 +700,8 @@ sq_status sq_scale_grad(sq_handle h, const sq_weight *w, const uint16_t *X, cons
   SQ_GUARD_END
 }
 
-// The handle's scratch on the current device, at least `bytes` (a larger buffer
-// replaces the old one; cudaFree waits for the work that may still use it). Growing
-// it is refused while `stream` is being captured into a graph (no allocation there).
 static sq_status ensure_workspace(sq_handle h, DeviceState *dev, size_t bytes, cudaStream_t stream) {
-  if (bytes <= dev->workspace_bytes) return SQ_OK;
-  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
-  cudaError_t e = cudaStreamIsCapturing(stream, &cap);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamIsCapturing");
-  if (cap != cudaStreamCaptureStatusNone)
-    return fail(h, SQ_ERR_UNSUPPORTED,
-                "the adapter kernels need %zu bytes of scratch: make one call outside graph capture first", bytes);
-  if (dev->workspace && (e = cudaFree(dev->workspace)) != cudaSuccess) return cuda_fail(h, e, "cudaFree(workspace)");
-  dev->workspace = nullptr;
-  dev->workspace_bytes = 0;
-  if ((e = cudaMalloc(&dev->workspace, bytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(workspace)");
-  dev->workspace_bytes = bytes;
-  return SQ_OK;
+  return ensure_scratch(h, dev->workspace, bytes, stream, "the adapter kernels");
 }
 
 static sq_status check_plane(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2) {
@@ -852,7 +869,7 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
   SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count), st));
-  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
+  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace.ptr),
                                dev->sm_count, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");
   return SQ_OK;
@@ -995,7 +1012,7 @@ sq_status sq_lowrank_product(sq_handle h, int64_t N, int64_t G, int32_t r, float
   SQ_TRY(check_buf(h, out, "out"));
   SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_product_workspace(N, G, r, dev->sm_count),
                           static_cast<cudaStream_t>(stream)));
-  cudaError_t e = sqi::launch_lowrank_product(N, G, r, alpha_over_r, B, A, out, static_cast<float *>(dev->workspace),
+  cudaError_t e = sqi::launch_lowrank_product(N, G, r, alpha_over_r, B, A, out, static_cast<float *>(dev->workspace.ptr),
                                               dev->sm_count, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(h, e, "low-rank product launch");
   return SQ_OK;
@@ -1134,7 +1151,7 @@ sq_status sq_grouped_lowrank_grad(sq_handle h, int32_t E, int64_t N, int64_t G, 
   SQ_TRY(check_buf(h, B, "B"));
   SQ_TRY(check_buf(h, A, "A"));
   SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count, E), st));
-  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace),
+  e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace.ptr),
                                dev->sm_count, st, E);
   if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter gradient launch");
   return SQ_OK;

@@ -37,17 +37,18 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 struct NoAllocDevice {
   bool ready;
   int sm_count;
-  int *scratch;  // device address of g_noalloc_scratch on this device
 };
 
 std::mutex g_mu;
 NoAllocDevice g_dev[kMaxDevices];
 EncodeTiledFn g_encode = nullptr;
 
-// Once per device, with that device current: check it and look up the device
-// address of the static scratch array (in host code its name is only a host-side
-// stand-in, so the kernel must be given this address).
-sq_status setup_current_device(NoAllocDevice **out) {
+// With the caller's device current: check it once (compute capability 10.3, SM
+// count, the driver's tensor-map encoder), then on every call look up the device
+// address of the static scratch array. In host code the array's name is only a
+// host-side stand-in, so the kernel must be given this address; looking it up
+// each time (it allocates nothing) keeps it right after a device reset.
+sq_status setup_current_device(NoAllocDevice **out, int **scratch) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return SQ_ERR_DEVICE;
   if (dev >= kMaxDevices) return SQ_ERR_UNSUPPORTED;
@@ -69,13 +70,13 @@ sq_status setup_current_device(NoAllocDevice **out) {
         return SQ_ERR_DEVICE;
       g_encode = reinterpret_cast<EncodeTiledFn>(fn);
     }
-    int *ptr = nullptr;
-    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&ptr), g_noalloc_scratch) != cudaSuccess || !ptr)
-      return SQ_ERR_CUDA;
-    d.scratch = ptr;
     d.sm_count = sms;
     d.ready = true;
   }
+  int *ptr = nullptr;
+  if (cudaGetSymbolAddress(reinterpret_cast<void **>(&ptr), g_noalloc_scratch) != cudaSuccess || !ptr)
+    return SQ_ERR_CUDA;
+  *scratch = ptr;
   *out = &d;
   return SQ_OK;
 }
@@ -110,13 +111,14 @@ extern "C" sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X
   if (kScratchNeeded > kScratchBytes) return SQ_ERR_INVALID_ARG;
 
   NoAllocDevice *dev = nullptr;
-  sq_status st = setup_current_device(&dev);
+  int *scratch = nullptr;
+  sq_status st = setup_current_device(&dev, &scratch);
   if (st != SQ_OK) return st;
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int B = w->fmt == SQ_NVFP4 ? 16 : 32;
 
   // The shared array keeps the last call's contents: clear the error word first.
-  if (cudaMemsetAsync(dev->scratch, 0, kScratchNeeded, s) != cudaSuccess) return SQ_ERR_CUDA;
+  if (cudaMemsetAsync(scratch, 0, kScratchNeeded, s) != cudaSuccess) return SQ_ERR_CUDA;
   if (M == 0) {
     if (cudaMemsetAsync(g, 0, static_cast<size_t>(w->N) * (w->K / B) * sizeof(float), s) != cudaSuccess)
       return SQ_ERR_CUDA;
@@ -134,11 +136,11 @@ extern "C" sq_status sq_scale_grad_noalloc(const sq_weight *w, const uint16_t *X
     a.ws2 = w->ws2;
     a.out = g;
     a.mask = mask;
-    a.err = dev->scratch;
+    a.err = scratch;
     if (sqi::launch_gemm(a, tmA, tmB, nullptr, dev->sm_count, s) != cudaSuccess) return SQ_ERR_CUDA;
   }
   if (device_status &&
-      cudaMemcpyAsync(device_status, dev->scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+      cudaMemcpyAsync(device_status, scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
     return SQ_ERR_CUDA;
   return SQ_OK;
 }
