@@ -579,12 +579,13 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
 // epilogue warps (two per TMEM lane quadrant, one per column half) shorten that
 // wait.
 struct PairCfg {
-  static constexpr int kEpiWarps = 8;    // warps 0-7: warp w drains lane quadrant w % 4, column half w / 4
-  static constexpr int kDecWarps = 16;   // warps 8-23: one 32-weight unit per thread per stage
+  // Roles are numbered 0-27 as below; role_of() places them on the physical warps.
+  static constexpr int kEpiWarps = 8;    // roles 0-7: warp w drains lane quadrant w % 4, column half w / 4
+  static constexpr int kDecWarps = 16;   // roles 8-23: one 32-weight unit per thread per stage
   static constexpr int kTmaWarp = kEpiWarps + kDecWarps;  // activation tiles
   static constexpr int kCodeWarp = kTmaWarp + 1;          // packed-code tiles
   static constexpr int kMmaWarp = kCodeWarp + 1;
-  static constexpr int kGateWarp = kMmaWarp + 1;  // leader: folds "decoded" and "activations landed" into one barrier
+  static constexpr int kGateWarp = kMmaWarp + 1;  // leader: hands each k-step to the MMA thread
   static constexpr int kThreads = 32 * (kGateWarp + 1);
   static constexpr int kBK = 128;        // contraction depth of a stage: 8 MMAs of K = 16 per tile half
   static constexpr int kAStages = 4;     // activation slots (two per k-step)
@@ -608,6 +609,32 @@ static_assert(PairCfg::kSmemBytes <= 232448, "pair kernel exceeds the opt-in sha
 static_assert(PairCfg::kMTile == 2 * PairCfg::kTile, "a pair tile is two halves");
 static_assert(PairCfg::kAStages == 2 * PairCfg::kStages, "half 1's activation slots are released with the decoded slots");
 static_assert(PairCfg::kEpiWarps == 8, "the epilogue maps warp w to lane quadrant w % 4 and column half w / 4");
+
+// Role of physical warp pw. Warp pw issues from scheduler pw % 4, and a
+// tcgen05.mma holds the MMA thread until the tensor core takes it, so every cycle
+// that thread waits for an issue slot can idle the tensor core. The MMA warp
+// (physical 26) therefore shares its scheduler with the two TMA warps (physical 18
+// and 22, mostly asleep on barriers), two epilogue warps and only two decode warps;
+// the decode roles fill physical 8-17, 19-21 and 23-25 and the gate stays on 27.
+// Measured against the plain numbering (the MMA warp beside four decode warps):
+// the MMA thread's 8 MMAs of a tile half issued in ~750 instead of ~1,030 cycles.
+// The epilogue roles keep their warps: TMEM lane quadrant access is by warp % 4.
+__device__ __forceinline__ int pair_role_of(int pw) {
+  switch (pw) {
+    case 18: return PairCfg::kCodeWarp;
+    case 22: return PairCfg::kTmaWarp;
+    case 19: return 18;
+    case 20: return 19;
+    case 21: return 20;
+    case 23: return 21;
+    case 24: return 22;
+    case 25: return 23;
+    default: return pw;
+  }
+}
+static_assert(PairCfg::kTmaWarp == 24 && PairCfg::kCodeWarp == 25 && PairCfg::kMmaWarp == 26 &&
+                  PairCfg::kGateWarp == 27,
+              "pair_role_of places these roles");
 
 // Decode unit u (0..511) of this CTA's half at stage kb covers 32 consecutive
 // weights: row (u & 7) + 8 * (u >> 5) of the half, quarter (u >> 3) & 3 of its
@@ -641,7 +668,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   uint64_t *empty = aempty + SA;      // [S] pair MMAs of k-step s done: decoded slot s and
                                       //     half 1's activation slot free      (multicast commit)
   uint64_t *pready = empty + S;       // [S] leader: both weight halves decoded          (1 arrival + st.async tx)
-  uint64_t *gready = pready + S;      // [S] leader: pready and both halves' afull seen by the gate (1 arrival)
+  uint64_t *gready = pready + S;      // [S] leader: pready and half 0's afull seen by the gate (1 arrival)
   uint64_t *cfull = gready + S;       // [SC] this CTA's code tile landed                 (1 arrival + tx)
   uint64_t *cempty = cfull + SC;      // [SC] this CTA's decode warps read the codes      (kDecWarps arrivals)
   uint64_t *tfull = cempty + SC;      // [2] accumulator h of the tile complete          (multicast commit)
@@ -652,7 +679,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   uint32_t *sink = reinterpret_cast<uint32_t *>(drain + 2);  // leader: st.async targets, [2][kDecWarps] + [kEpiWarps]
 
-  const int warp = threadIdx.x >> 5;
+  const int warp = pair_role_of(threadIdx.x >> 5);  // this warp's role
   const int lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const int cluster = blockIdx.x >> 1;
@@ -802,12 +829,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
   } else if (warp == C::kMmaWarp) {
     // ------------------------------------------------------ MMA issuer (leader CTA)
     // A k-step needs both decoded weight halves and the activation tiles of both
-    // halves, which the gate warp folds into one barrier (gready). Every barrier
-    // wait and every commit of this thread costs issue time the tensor core cannot
-    // hide, so it waits once per k-step, spinning (test_wait), polls nothing between
-    // MMAs and commits twice: half 0's activation slot after its 8 MMAs (the TMA
-    // warp refills it a half step early) and, after all 16, the decoded slot together
-    // with half 1's activation slot.
+    // halves. The gate warp folds the decoded halves and half 0's activations into
+    // one barrier (gready); half 1's activations, whose slot is refilled last, are
+    // checked here just before half 1's MMAs, which gives their loads half a k-step
+    // more time. Every barrier wait and every commit of this thread costs issue time
+    // the tensor core cannot hide, so it waits spinning (test_wait), polls nothing
+    // between MMAs and commits twice: half 0's activation slot after its 8 MMAs (the
+    // TMA warp refills it a half step early) and, after all 16, the decoded slot
+    // together with half 1's activation slot.
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_bf16(2 * 128, C::kTile, 0, MODE == MODE_FWD ? 0 : 1);
       // slot s of a ring starts s slot sizes after slot 0 (the start address field is >> 4).
@@ -826,6 +855,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
+            // half 1's activation tiles landed
+            if (h == 1 && !(ok = mbar_spin(&afull[a], static_cast<uint32_t>((2 * it + 1) / SA) & 1u, abort_flag, p.err)))
+              break;
             // the previous tile's epilogue has drained accumulator h
             if (kb == 0 && tc >= 1 &&
                 !(ok = mbar_spin_cluster(&tempty[h], static_cast<uint32_t>(tc - 1) & 1u, abort_flag, p.err)))
@@ -856,20 +888,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     }
   } else if (warp == C::kGateWarp) {
     // ------------------------------------------------------ gate (leader CTA)
-    // Waits, for each k-step, for both decoded halves (pready, a cluster-scope
-    // acquire that costs a few hundred cycles even on a completed barrier) and for
-    // the activation tiles of both halves (afull), then hands the step to the MMA thread
-    // through one CTA-local barrier. It also arms pready with the signal
-    // bytes of each use (decode warps may signal before it is armed: the missing
-    // arrival keeps the phase open).
+    // Waits, for each k-step, for half 0's activation tiles (afull; they usually
+    // land first) and then for both decoded halves (pready, a cluster-scope acquire
+    // that costs a few hundred cycles even on a completed barrier), and hands the
+    // step to the MMA thread through one CTA-local barrier. It also arms pready with
+    // the signal bytes of each use (decode warps may signal before it is armed: the
+    // missing arrival keeps the phase open).
     if (lane == 0 && rank == 0) {
       const int iters = my_tiles * num_k;
       for (int s = 0; s < S && s < iters; ++s) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       for (int it = 0; it < iters; ++it) {
         const int s = it % S;
-        if (!mbar_spin_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
         if (!mbar_spin(&afull[(2 * it) % SA], static_cast<uint32_t>((2 * it) / SA) & 1u, abort_flag, p.err)) break;
-        if (!mbar_spin(&afull[(2 * it + 1) % SA], static_cast<uint32_t>((2 * it + 1) / SA) & 1u, abort_flag, p.err)) break;
+        if (!mbar_spin_cluster(&pready[s], static_cast<uint32_t>(it / S) & 1u, abort_flag, p.err)) break;
         mbar_arrive(&gready[s]);
         if (it + S < iters) mbar_arrive_expect_tx(&pready[s], C::kSignalBytes);
       }
@@ -996,10 +1027,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
 #pragma unroll
       for (int d = 0; d < kD; ++d) {
         if (cur.tile >= total || !ok) break;
-        if (lane == 0) {
-          ok = mbar_wait(&cfull[cs], cph, abort_flag, p.err);
-          if (ok && it >= S) ok = mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.err);
-        }
+        // The stage is decoded into registers as soon as its codes land; only the
+        // stores wait for the decoded slot (freed by the MMAs of k-step it - S), and
+        // that wait spins, so the slot is refilled within a few hundred cycles of
+        // its release (the slot's round trip bounds the k-step rate).
+        if (lane == 0) ok = mbar_wait(&cfull[cs], cph, abort_flag, p.err);
         ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
         __syncwarp();
         if (!ok) break;
@@ -1011,21 +1043,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           sc_lo = sc_hi = scale_bf16x2<1>(sc[d]);
         }
         const uint4 cw = lds128(smem_u32(ring_c(cs)) + c_off);
-        const uint32_t b_base = smem_u32(ring_b(s));
         const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+        uint32_t o[4][4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-          uint32_t o[4];
-          e2m1x8_to_bf16(words[c], o);
+          e2m1x8_to_bf16(words[c], o[c]);
           const uint32_t scv = c < 2 ? sc_lo : sc_hi;
 #pragma unroll
-          for (int q = 0; q < 4; ++q) o[q] = bf16x2_mul(o[q], scv);
-          st_shared_v4(b_base + b_off[c], o[0], o[1], o[2], o[3]);
+          for (int q = 0; q < 4; ++q) o[c][q] = bf16x2_mul(o[c][q], scv);
         }
-        fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&cempty[cs]);  // the warp's code reads are done
+          if (it >= S) ok = mbar_spin(&empty[s], ph ^ 1u, abort_flag, p.err);
+        }
+        ok = __shfl_sync(0xFFFFFFFFu, ok ? 1 : 0, 0) != 0;
+        __syncwarp();
+        if (!ok) break;
+        const uint32_t b_base = smem_u32(ring_b(s));
+#pragma unroll
+        for (int c = 0; c < 4; ++c) st_shared_v4(b_base + b_off[c], o[c][0], o[c][1], o[c][2], o[c][3]);
+        fence_proxy_async_smem();  // this thread's shared-memory writes -> async proxy
+        __syncwarp();
+        if (lane == 0) {
           // tell the leader without waiting: an async store whose complete-tx on the
           // leader's stage barrier is a cluster-scope release (both CTAs, all decode warps)
           st_async_signal(sink_addr, mapa_shared(smem_u32(&pready[s]), 0));
