@@ -49,6 +49,9 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="c5")
+    ap.add_argument("--linears", default=None,
+                    help="comma-separated subset of the workload's linears (e.g. q_proj): the step runs only "
+                         "these; for profiling one linear of the layer on a few GB of device memory")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-context", action="store_true",
@@ -256,7 +259,8 @@ class LayerState:
         self.wl = wl
         self.lowrank = lowrank
         self.lin = []
-        self.acts = {name: synth.gen_act(wl, name, device=device) for name in synth.act_names(wl)}
+        self.acts = {name: synth.gen_act(wl, name, device=device) for name in synth.act_names(wl)
+                     if any(l.x == name for l in wl.linears)}
         for lin in wl.linears:
             w = synth.gen_weight(wl, lin, device=device)
             L = synth.gen_latent(wl, lin, w, device=device)
@@ -773,6 +777,13 @@ def run_ours(args):
     torch.cuda.set_device(local)
     build.build()
     wl = synth.WORKLOADS[args.workload]
+    if args.linears:
+        import dataclasses
+        keep = args.linears.split(",")
+        wl = dataclasses.replace(wl, linears=tuple(l for l in wl.linears if l.name in keep),
+                                 title=f"{wl.title}, only {args.linears}")
+        if not wl.linears:
+            raise SystemExit(f"--linears {args.linears}: no such linear in {args.workload}")
     pk = peaks()
     h = pkg.Handle()
     stream = torch.cuda.current_stream()
@@ -841,7 +852,7 @@ def run_ours(args):
                                                   else DATASHEET["hbm_gbs"])
     per_ghz(kernels, clk)
     dom = max(("fwd", "dx", "sgrad"), key=lambda k: kind_ms[k])
-    traffic = {} if args.lowrank else profiled_traffic(wl.key)  # the profile is of the default step's kernels
+    traffic = {} if (args.lowrank or args.linears) else profiled_traffic(wl.key)  # the profile is of the default step's kernels
     for kind in kinds:
         if kind in traffic:
             kernels[kind]["dram_bytes_per_launch"] = traffic[kind]["dram_bytes_per_launch"]
