@@ -309,50 +309,66 @@ def flat_inputs(ins):
     return list(ins["acts"].values()) + ins["dY"] + ins["L"]
 
 
-def run_step(h, S, stream, events=None, ins=None):
-    """One step over every linear: projection (+ STE mask), forward, input gradient,
-    masked scale gradient, merge into the artifact scale plane. With the low-rank
-    adapter (S.lowrank) the latent is formed from the adapter inside the projection
-    (and kept for the merge), and the adapter gradients follow the scale gradient."""
+def run_step(h, S, stream, timer=None, ins=None):
+    """One step over every linear: grid projection (+ STE mask) of all linears' latents
+    in one launch, then per linear the forward, input gradient and masked scale
+    gradient, and the merge of all latents into the artifact scale planes in one
+    launch. With the low-rank adapter (S.lowrank) each linear's latent is formed from
+    its adapter inside its projection (and kept for the merge), and the adapter
+    gradients follow the scale gradient. `timer(kind)` records an event after each
+    kind's launch(es)."""
     fmt = S.wl.fmt
     ins = input_set(S) if ins is None else ins
+    mark = timer if timer is not None else (lambda kind: None)
+    mark(None)
+    if S.lowrank:
+        for i, st in enumerate(S.lin):
+            h.sq_project_lowrank(fmt, st["base_scales"], st["B"], st["A"], st["ws2"], st["aor"],
+                                 bytes_out=st["qbytes"], mask_out=st["mask"], nonfinite=st["nonfinite"],
+                                 latent_out=ins["L"][i], stream=stream)
+    else:
+        h.sq_project_planes(fmt, [dict(latent=ins["L"][i], bytes=st["qbytes"], mask=st["mask"],
+                                       nonfinite=st["nonfinite"], ws2=st["ws2"]) for i, st in enumerate(S.lin)],
+                            stream=stream)
+    mark("project")
     for i, st in enumerate(S.lin):
         X = ins["acts"][st["lin"].x]
         dY = ins["dY"][i]
-        L = ins["L"][i]
-        ev = events[i] if events is not None else None
-        e = 0
-
-        def mark():
-            nonlocal e
-            if ev:
-                ev[e].record(stream)
-            e += 1
-
-        mark()
-        if S.lowrank:
-            h.sq_project_lowrank(fmt, st["base_scales"], st["B"], st["A"], st["ws2"], st["aor"],
-                                 bytes_out=st["qbytes"], mask_out=st["mask"], nonfinite=st["nonfinite"],
-                                 latent_out=L, stream=stream)
-        else:
-            h.sq_project_scales(fmt, L, st["ws2"], bytes_out=st["qbytes"], mask_out=st["mask"],
-                                nonfinite=st["nonfinite"], stream=stream)
-        mark()
         h.sq_fwd(st["qw"], X, st["Y"], stream=stream)
-        mark()
+        mark("fwd")
         h.sq_bwd_dx(st["qw"], dY, st["dX"], stream=stream)
-        mark()
+        mark("dx")
         h.sq_scale_grad(st["qw"], X, dY, mask=st["mask"], g=st["g"], stream=stream)
-        mark()
+        mark("sgrad")
         if S.lowrank:
             h.sq_lowrank_grad(st["g"], st["B"], st["A"], st["aor"], dB=st["dB"], dA=st["dA"], stream=stream)
-            mark()
-        h.sq_merge(fmt, L, st["ws2"], st["art"], changed=st["changed"], stream=stream)
-        mark()
+            mark("adapter_grad")
+    h.sq_merge_planes(fmt, [dict(latent=ins["L"][i], bytes=st["art"], changed=st["changed"], ws2=st["ws2"])
+                            for i, st in enumerate(S.lin)], stream=stream)
+    mark("merge")
 
 
-LAUNCHES_PER_LINEAR = 5  # project, fwd, dX, scale-grad, merge (+1 where the scale gradient splits its tokens)
-LAUNCHES_PER_LINEAR_LOWRANK = 9  # + the adapter gradients' four kernels (dB and dA products, each chunk sum)
+class StepTimer:
+    """CUDA events between the kinds of a step's launches, on the launching stream."""
+
+    def __init__(self, stream):
+        self.stream = stream
+        self.marks = []
+
+    def __call__(self, kind):
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(self.stream)
+        self.marks.append((kind, e))
+
+    def add_to(self, kind_ms, kind_launch):
+        for (_, a), (kind, b) in zip(self.marks[:-1], self.marks[1:]):
+            kind_ms[kind] += a.elapsed_time(b)
+            kind_launch[kind] += 1
+
+
+LAUNCHES_PER_STEP = 2    # the projection and the merge of all linears' planes
+LAUNCHES_PER_LINEAR = 3  # fwd, dX, scale-grad (+1 where the scale gradient splits its tokens)
+LAUNCHES_PER_LINEAR_LOWRANK = 8  # + the adapter projection and the adapter gradients' four kernels
 
 
 def kernel_work(S):
@@ -804,15 +820,14 @@ def run_ours(args):
 
     # ---- device-resident timed region (inputs already in HBM; inputs > L2)
     nl = len(S.lin)
-    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(len(kinds) + 1)] for _ in range(nl)]
-              for _ in range(args.steps)]
+    timers = [StepTimer(stream) for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     t_start.record(stream)
     for k in range(args.steps):
-        run_step(h, S, stream, events[k])
+        run_step(h, S, stream, timers[k])
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -830,12 +845,8 @@ def run_ours(args):
 
     kind_ms = {k: 0.0 for k in kinds}
     kind_launch = {k: 0 for k in kinds}
-    for k in range(args.steps):
-        for i in range(nl):
-            ev = events[k][i]
-            for j, kind in enumerate(kinds):
-                kind_ms[kind] += ev[j].elapsed_time(ev[j + 1])
-                kind_launch[kind] += 1
+    for t in timers:
+        t.add_to(kind_ms, kind_launch)
     fl, by = kernel_work(S)
     kernels = {}
     for kind in kinds:
@@ -950,7 +961,8 @@ def run_ours(args):
             "verified": verified,
             "kernels": kernels,
             "e2e": e2e, "cpu_baseline": cpu,
-            "gpu_launches": ((LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl
+            "gpu_launches": (LAUNCHES_PER_STEP - (1 if args.lowrank else 0)
+                             + (LAUNCHES_PER_LINEAR_LOWRANK if args.lowrank else LAUNCHES_PER_LINEAR) * nl
                              + sum(h.sq_scale_grad_workspace(st["qw"], S.wl.M)[0] > 1 for st in S.lin)) * args.steps,
             "clocks": clk,
         }

@@ -176,6 +176,43 @@ sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, floa
 sq_status sq_merge(sq_handle h, int32_t fmt, int64_t N, int64_t G, float ws2, const float *latent,
                    uint8_t *scales_inout, float *ongrid_delta, int64_t *changed_bytes, void *stream);
 
+/* One scale plane of a multi-plane call: the N x G blocks of one linear (layouts
+ * as above). N * G must be a multiple of 16 (it is for every linear: N % 8 == 0
+ * and G % 16 == 0). sq_project_planes uses latent, bytes (bytes_out), mask
+ * (nullable) and nonfinite (nullable, device int32); sq_merge_planes uses latent,
+ * bytes (the artifact's scale plane, in place), ongrid_delta (nullable) and
+ * changed_bytes (nullable, device int64). Fields a call does not use are ignored. */
+typedef struct {
+  int64_t N, G;
+  float ws2;                 /* NVFP4 tensor scale of this plane; 1.0f for MXFP4 */
+  const float *latent;       /* device fp32 [N, G] */
+  uint8_t *bytes;            /* device u8 [N, G] */
+  uint8_t *mask;             /* device u8 [N, G] or NULL */
+  float *ongrid_delta;       /* device fp32 [N, G] or NULL */
+  int32_t *nonfinite;        /* device int32 or NULL */
+  int64_t *changed_bytes;    /* device int64 or NULL */
+} sq_plane;
+#define SQ_MAX_PLANES 16
+
+/* The projection of sq_project_scales applied to up to SQ_MAX_PLANES planes of
+ * different shapes in ONE kernel launch (the scale planes of every linear of a
+ * layer, Sec. 3 QAST round_grid; bytes identical to one sq_project_scales call
+ * per plane). The plane table is copied into the launch's parameters (`planes` is
+ * a host array and may be reused as soon as the call returns); the call makes no
+ * allocation and no copy, so it can be captured into a CUDA graph. Each plane's
+ * counter receives its own NaN count. Uses a small counter accumulator of the
+ * handle (allocated with the handle's device state): calls of one handle must be
+ * ordered on the GPU. nplanes == 0 is a no-op. Returns SQ_ERR_INVALID_ARG for a bad
+ * plane (shape, alignment, ws2) before anything is launched. */
+sq_status sq_project_planes(sq_handle h, int32_t fmt, int32_t nplanes, const sq_plane *planes, void *stream);
+
+/* The merge of sq_merge (Sec. 3 "QAST makes merge exact by construction"; Sec. 5
+ * Payoff 3: one merge touches every target linear) over up to SQ_MAX_PLANES planes
+ * in ONE kernel launch, with the same table, counter and ordering rules as
+ * sq_project_planes; bytes, deltas and changed counts identical to one sq_merge
+ * call per plane. No code pointer is taken. */
+sq_status sq_merge_planes(sq_handle h, int32_t fmt, int32_t nplanes, const sq_plane *planes, void *stream);
+
 /* Rollback, Sec. 5 Payoff 3 ("invertible merges and rollback"): subtracting the
  * on-grid scale delta a merge applied restores the base plane byte for byte. In
  * place, every byte b of scales_inout becomes the projection (the merge's grid and

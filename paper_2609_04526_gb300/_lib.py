@@ -31,7 +31,7 @@ EXPORTS = ("sq_create", "sq_destroy", "sq_status_string", "sq_last_error", "sq_s
            "sq_grouped_bwd_dx", "sq_grouped_scale_grad", "sq_grouped_project_scales", "sq_grouped_merge",
            "sq_grouped_project_lowrank", "sq_grouped_lowrank_grad", "sq_fit_scale_delta", "sq_group_reduce",
            "sq_project_group_delta", "sq_control_fwd", "sq_control_bwd_dx", "sq_control_grad", "sq_lowrank_product",
-           "sq_selftest_wait_timeout", "sq_scale_grad_workspace")
+           "sq_selftest_wait_timeout", "sq_scale_grad_workspace", "sq_project_planes", "sq_merge_planes")
 
 
 class SQError(RuntimeError):
@@ -82,6 +82,8 @@ def load() -> ctypes.CDLL:
     L.sq_scale_grad.argtypes = [vp, W, vp, vp, i64, vp, vp, vp]
     L.sq_project_scales.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
     L.sq_merge.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp, vp]
+    L.sq_project_planes.argtypes = [vp, i32, i32, ctypes.POINTER(_SqPlane), vp]
+    L.sq_merge_planes.argtypes = [vp, i32, i32, ctypes.POINTER(_SqPlane), vp]
     L.sq_project_lowrank.argtypes = [vp, i32, i64, i64, i32, f32, f32, vp, vp, vp, vp, vp, vp, vp, vp]
     L.sq_lowrank_grad.argtypes = [vp, i64, i64, i32, f32, vp, vp, vp, vp, vp, vp]
     L.sq_rollback.argtypes = [vp, i32, i64, i64, f32, vp, vp, vp, vp]
@@ -109,6 +111,12 @@ def load() -> ctypes.CDLL:
             getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
+
+
+class _SqPlane(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int64), ("G", ctypes.c_int64), ("ws2", ctypes.c_float), ("latent", ctypes.c_void_p),
+                ("bytes", ctypes.c_void_p), ("mask", ctypes.c_void_p), ("ongrid_delta", ctypes.c_void_p),
+                ("nonfinite", ctypes.c_void_p), ("changed_bytes", ctypes.c_void_p)]
 
 
 @dataclasses.dataclass
@@ -318,6 +326,27 @@ class Handle:
         self._check(self._L.sq_merge(self._h, fmt, N, G, ws2, _ptr(latent), _ptr(scales_inout), _ptr(ongrid_delta),
                                      _ptr(changed), _stream(stream)))
         return scales_inout
+
+    def _planes(self, planes):
+        arr = (_SqPlane * max(1, len(planes)))()
+        for i, p in enumerate(planes):
+            N, G = p["latent"].shape
+            arr[i] = _SqPlane(N, G, float(p.get("ws2", 1.0)), _ptr(p["latent"]), _ptr(p["bytes"]), _ptr(p.get("mask")),
+                              _ptr(p.get("ongrid_delta")), _ptr(p.get("nonfinite")), _ptr(p.get("changed")))
+        return arr
+
+    def sq_project_planes(self, fmt: int, planes, stream=None):
+        """One launch for several planes: planes is a list of dicts with latent [N, G]
+        fp32, bytes [N, G] u8 (out), and optional ws2, mask (out), nonfinite (int32 [1])."""
+        arr = self._planes(planes)
+        self._check(self._L.sq_project_planes(self._h, fmt, len(planes), arr, _stream(stream)))
+
+    def sq_merge_planes(self, fmt: int, planes, stream=None):
+        """One launch for several planes: planes is a list of dicts with latent [N, G]
+        fp32, bytes [N, G] u8 (the scale plane, in place), and optional ws2,
+        ongrid_delta [N, G] fp32, changed (int64 [1])."""
+        arr = self._planes(planes)
+        self._check(self._L.sq_merge_planes(self._h, fmt, len(planes), arr, _stream(stream)))
 
     # experts of an MoE linear ------------------------------------------------
     def sq_grouped_fwd(self, w: GroupedWeight, offsets, X: torch.Tensor, Y: Optional[torch.Tensor] = None,

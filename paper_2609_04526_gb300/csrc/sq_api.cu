@@ -49,6 +49,7 @@ struct DeviceState {
   TableSlot tables[kTableSlots];
   int next_table;
   Scratch partial;       // token-split partial planes of the dense scale gradient
+  int64_t *plane_acc;    // counter accumulators of the multi-plane calls (zero between calls)
 };
 
 constexpr int64_t kMaxDim = int64_t(1) << 24;       // N, K limit
@@ -111,10 +112,14 @@ sq_status ensure_device(sq_handle h, DeviceState **out) {
   int *err_word = nullptr;
   if ((e = cudaMalloc(&err_word, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(error word)");
   if ((e = cudaMemset(err_word, 0, sizeof(int))) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(error word)");
+  int64_t *plane_acc = nullptr;
+  if ((e = cudaMalloc(&plane_acc, sqi::kPlaneAccBytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(plane counters)");
+  if ((e = cudaMemset(plane_acc, 0, sqi::kPlaneAccBytes)) != cudaSuccess) return cuda_fail(h, e, "cudaMemset(plane counters)");
   DeviceState d{};
   d.device = dev;
   d.sm_count = sms;
   d.err_word = err_word;
+  d.plane_acc = plane_acc;
   d.next_table = 0;
   h->devices.push_back(std::move(d));
   *out = &h->devices.back();
@@ -576,6 +581,7 @@ sq_status sq_destroy(sq_handle h) {
   for (auto &d : h->devices) {
     if (cudaSetDevice(d.device) == cudaSuccess) {
       cudaFree(d.err_word);
+      if (d.plane_acc) cudaFree(d.plane_acc);
       free_scratch(d.workspace);
       free_scratch(d.partial);
       for (auto &t : d.tables) {
@@ -726,6 +732,67 @@ sq_status sq_project_scales(sq_handle h, int32_t fmt, int64_t N, int64_t G, floa
   cudaError_t e = sqi::launch_project(fmt, N * G, ws2, latent, bytes_out, mask_out, nonfinite, dev->sm_count,
                                       static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(h, e, "projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+// Checks the plane table of a multi-plane call and fills the kernel's copy.
+static sq_status planes_table(sq_handle h, int32_t fmt, int32_t nplanes, const sq_plane *planes, bool merge,
+                              sqi::PlaneTable *t) {
+  if (nplanes < 0 || nplanes > sqi::kMaxPlanes)
+    return fail(h, SQ_ERR_INVALID_ARG, "nplanes=%d out of range [0, %d]", nplanes, sqi::kMaxPlanes);
+  if (nplanes > 0 && !planes) return fail(h, SQ_ERR_INVALID_ARG, "planes is NULL");
+  t->n = nplanes;
+  for (int j = 0; j < nplanes; ++j) {
+    const sq_plane &p = planes[j];
+    SQ_TRY(check_plane(h, fmt, p.N, p.G, p.ws2));
+    if ((p.N * p.G) % 16 != 0)
+      return fail(h, SQ_ERR_INVALID_ARG, "plane %d: N * G = %lld is not a multiple of 16", j, (long long)(p.N * p.G));
+    SQ_TRY(check_buf(h, p.latent, "plane latent"));
+    SQ_TRY(check_buf(h, p.bytes, merge ? "plane scales" : "plane bytes"));
+    if (!merge && p.mask && !aligned16(p.mask)) return fail(h, SQ_ERR_INVALID_ARG, "plane %d: mask must be 16-byte aligned", j);
+    if (merge && p.ongrid_delta && !aligned16(p.ongrid_delta))
+      return fail(h, SQ_ERR_INVALID_ARG, "plane %d: ongrid_delta must be 16-byte aligned", j);
+    if (!merge && p.nonfinite && (reinterpret_cast<uintptr_t>(p.nonfinite) & 3u))
+      return fail(h, SQ_ERR_INVALID_ARG, "plane %d: nonfinite must be 4-byte aligned", j);
+    if (merge && p.changed_bytes && (reinterpret_cast<uintptr_t>(p.changed_bytes) & 7u))
+      return fail(h, SQ_ERR_INVALID_ARG, "plane %d: changed_bytes must be 8-byte aligned", j);
+    sqi::PlaneArgs &a = t->p[j];
+    a.count = p.N * p.G;
+    a.ws2 = p.ws2;
+    a.latent = p.latent;
+    a.bytes = p.bytes;
+    a.mask = merge ? nullptr : p.mask;
+    a.delta = merge ? p.ongrid_delta : nullptr;
+    a.counter = merge ? static_cast<void *>(p.changed_bytes) : static_cast<void *>(p.nonfinite);
+  }
+  return SQ_OK;
+}
+
+sq_status sq_project_planes(sq_handle h, int32_t fmt, int32_t nplanes, const sq_plane *planes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  sqi::PlaneTable t{};
+  SQ_TRY(planes_table(h, fmt, nplanes, planes, false, &t));
+  if (nplanes == 0) return SQ_OK;
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_project_planes(fmt, t, dev->plane_acc, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "multi-plane projection launch");
+  return SQ_OK;
+  SQ_GUARD_END
+}
+
+sq_status sq_merge_planes(sq_handle h, int32_t fmt, int32_t nplanes, const sq_plane *planes, void *stream) {
+  if (!h) return SQ_ERR_INVALID_ARG;
+  SQ_GUARD_BEGIN
+  sqi::PlaneTable t{};
+  SQ_TRY(planes_table(h, fmt, nplanes, planes, true, &t));
+  if (nplanes == 0) return SQ_OK;
+  DeviceState *dev = nullptr;
+  SQ_TRY(ensure_device(h, &dev));
+  cudaError_t e = sqi::launch_merge_planes(fmt, t, dev->plane_acc, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "multi-plane merge launch");
   return SQ_OK;
   SQ_GUARD_END
 }

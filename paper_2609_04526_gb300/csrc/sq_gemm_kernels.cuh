@@ -978,7 +978,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // ------------------------------------------------------ decode (both CTAs)
     // Every decode thread turns one 32-weight unit of every stage into bf16:
     // codes from the code ring, into the decoded slot the MMAs of k-step it - S freed.
-    constexpr int kD = SQ_SCALE_DEPTH;
+    // (grouped launches keep per-expert tile state in the decode warps: a shallower scale
+    // prefetch keeps them within the 72 registers without spilling)
+    constexpr int kD = GR ? 2 : SQ_SCALE_DEPTH;
     const int dw = warp - C::kEpiWarps;
     const int u = dw * 32 + lane;  // this thread's unit, 0..511
     struct Pos {

@@ -131,6 +131,29 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
                          float *ongrid_delta, int64_t *changed, int sm_count, cudaStream_t stream,
                          const float *ws2_per = nullptr, int64_t plane = 0);
 
+// Projection / merge of several scale planes of different shapes in one launch
+// (the planes of all linears of a layer). The table travels by value in the
+// kernel's parameters; each plane's N * G is a multiple of 16. Counters are summed
+// per CTA into `acc` (kMaxPlanes int64 plus a uint32 ticket, zero between calls:
+// the last CTA writes each plane's count to its counter and clears them).
+constexpr int kMaxPlanes = 16;
+struct PlaneArgs {
+  int64_t count;     // scale blocks (N * G)
+  float ws2;         // NVFP4 tensor scale (1 for MXFP4)
+  const float *latent;
+  uint8_t *bytes;    // projection: bytes out; merge: the scale plane, in place
+  uint8_t *mask;     // projection: mask out or null
+  float *delta;      // merge: on-grid delta or null
+  void *counter;     // projection: int32 NaN count; merge: int64 changed bytes; or null
+};
+struct PlaneTable {
+  int n;
+  PlaneArgs p[kMaxPlanes];
+};
+constexpr size_t kPlaneAccBytes = kMaxPlanes * sizeof(int64_t) + 16;
+cudaError_t launch_project_planes(int fmt, const PlaneTable &t, int64_t *acc, cudaStream_t stream);
+cudaError_t launch_merge_planes(int fmt, const PlaneTable &t, int64_t *acc, cudaStream_t stream);
+
 // Rollback of a merge by its on-grid delta (in place, counting changed bytes), and
 // copy a -> b (write) or only count the bytes in which a and b differ.
 cudaError_t launch_rollback(int fmt, int64_t count, float ws2, const float *delta, uint8_t *scales_inout,

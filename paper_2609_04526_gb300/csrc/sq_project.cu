@@ -230,6 +230,154 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
   if (changed) warp_add_i64(changed, n_changed);
 }
 
+// ---------------------------------------------------------------- several planes per launch
+//
+// The planes of all linears of a layer (Sec. 5 Payoff 3: the merge touches every
+// target linear) in one launch each for projection and merge. Every CTA works on
+// kPlaneVecs 16-element vectors of one plane (the CTAs of plane j follow those of
+// plane j - 1), so it reduces its counter within the block and adds it with one
+// atomic; the last CTA to finish (a ticket) writes every plane's count and clears
+// the accumulators for the next call.
+constexpr int kPlaneVecsPerThread = 4;
+constexpr int kPlaneVecs = kThreads * kPlaneVecsPerThread;
+
+__device__ __forceinline__ int plane_of_block(const PlaneTable &t, int64_t b, int64_t &first_block) {
+  int64_t start = 0;
+  for (int j = 0; j < t.n; ++j) {
+    const int64_t nb = (t.p[j].count / 16 + kPlaneVecs - 1) / kPlaneVecs;
+    if (b < start + nb) {
+      first_block = start;
+      return j;
+    }
+    start += nb;
+  }
+  first_block = start;
+  return t.n;  // not reached: the grid covers the planes exactly
+}
+
+// Block sum of v; the result is valid in thread 0.
+__device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t *red) {
+  v = __reduce_add_sync(0xFFFFFFFFu, v);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  uint32_t s = 0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < kThreads / 32; ++w) s += red[w];
+  return s;
+}
+
+// Adds this CTA's count of plane j to acc[j]; the last CTA writes the totals to the
+// planes' counters (int32 for the projection, int64 for the merge) and clears acc.
+template <bool I64>
+__device__ __forceinline__ void plane_counters(const PlaneTable &t, int j, uint32_t mine, int64_t *acc,
+                                               uint32_t *red) {
+  const uint32_t s = block_sum(mine, red);
+  if (threadIdx.x != 0) return;
+  if (s) atomicAdd(reinterpret_cast<unsigned long long *>(acc + j), static_cast<unsigned long long>(s));
+  __threadfence();
+  unsigned int *ticket = reinterpret_cast<unsigned int *>(acc + kMaxPlanes);
+  if (atomicAdd(ticket, 1u) != gridDim.x - 1) return;
+  __threadfence();
+  for (int q = 0; q < t.n; ++q) {
+    const unsigned long long v = atomicExch(reinterpret_cast<unsigned long long *>(acc + q), 0ull);
+    if (t.p[q].counter) {
+      if (I64)
+        *static_cast<int64_t *>(t.p[q].counter) = static_cast<int64_t>(v);
+      else
+        *static_cast<int32_t *>(t.p[q].counter) = static_cast<int32_t>(v);
+    }
+  }
+  *ticket = 0u;
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
+                                                                     int64_t *acc) {
+  __shared__ uint32_t red[kThreads / 32];
+  int64_t first_block;
+  const int j = plane_of_block(t, blockIdx.x, first_block);
+  const PlaneArgs &pl = t.p[j];
+  const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;  // the same IEEE fp32 product as the single-plane cap
+  const int64_t nvec = pl.count / 16;
+  const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
+  uint32_t nan_count = 0;
+#pragma unroll
+  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
+    const int64_t v = v0 + r * kThreads;
+    if (v >= nvec) break;
+    const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
+    float L[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 f = __ldcs(src + q);
+      L[4 * q] = f.x;
+      L[4 * q + 1] = f.y;
+      L[4 * q + 2] = f.z;
+      L[4 * q + 3] = f.w;
+    }
+    uint32_t ob[4] = {0, 0, 0, 0}, om[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      uint32_t b, m, n;
+      project_one<FMT>(L[i], ws2, cap, b, m, n);
+      ob[i >> 2] |= b << (8 * (i & 3));
+      om[i >> 2] |= m << (8 * (i & 3));
+      nan_count += n;
+    }
+    __stcs(reinterpret_cast<uint4 *>(pl.bytes) + v, make_uint4(ob[0], ob[1], ob[2], ob[3]));
+    if (pl.mask) __stcs(reinterpret_cast<uint4 *>(pl.mask) + v, make_uint4(om[0], om[1], om[2], om[3]));
+  }
+  plane_counters<false>(t, j, nan_count, acc, red);
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads) sq_merge_planes_kernel(const __grid_constant__ PlaneTable t,
+                                                                   int64_t *acc) {
+  __shared__ uint32_t red[kThreads / 32];
+  int64_t first_block;
+  const int j = plane_of_block(t, blockIdx.x, first_block);
+  const PlaneArgs &pl = t.p[j];
+  const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;
+  const int64_t nvec = pl.count / 16;
+  const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
+  uint32_t n_changed = 0;
+#pragma unroll
+  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
+    const int64_t v = v0 + r * kThreads;
+    if (v >= nvec) break;
+    const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
+    float L[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 f = __ldcs(src + q);
+      L[4 * q] = f.x;
+      L[4 * q + 1] = f.y;
+      L[4 * q + 2] = f.z;
+      L[4 * q + 3] = f.w;
+    }
+    const uint4 old4 = *(reinterpret_cast<const uint4 *>(pl.bytes) + v);
+    const uint32_t old[4] = {old4.x, old4.y, old4.z, old4.w};
+    uint32_t ob[4] = {0, 0, 0, 0};
+    float d[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      uint32_t b, m, n;
+      project_one<FMT>(L[i], ws2, cap, b, m, n);
+      const uint32_t o = (old[i >> 2] >> (8 * (i & 3))) & 0xFFu;
+      ob[i >> 2] |= b << (8 * (i & 3));
+      n_changed += (b != o) ? 1u : 0u;
+      d[i] = __fsub_rn(scale_value<FMT>(b, ws2), scale_value<FMT>(o, ws2));
+    }
+    *(reinterpret_cast<uint4 *>(pl.bytes) + v) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+    if (pl.delta) {
+      float4 *dst = reinterpret_cast<float4 *>(pl.delta) + 4 * v;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) __stcs(dst + q, make_float4(d[4 * q], d[4 * q + 1], d[4 * q + 2], d[4 * q + 3]));
+    }
+  }
+  plane_counters<true>(t, j, n_changed, acc, red);
+}
+
 // ---------------------------------------------------------------- rollback, swap, audit
 //
 // Sec. 5 Payoff 3: a merge is undone by subtracting the on-grid delta it applied;
@@ -806,6 +954,46 @@ cudaError_t launch_merge(int fmt, int64_t count, float ws2, const float *latent,
   else
     sq_merge_kernel<1, false><<<grid, kThreads, 0, stream>>>(count, ws2, cap, nullptr, 0, latent, scales_inout,
                                                              ongrid_delta, changed);
+  return cudaGetLastError();
+}
+
+static unsigned planes_grid(const PlaneTable &t) {
+  int64_t g = 0;
+  for (int j = 0; j < t.n; ++j) g += (t.p[j].count / 16 + kPlaneVecs - 1) / kPlaneVecs;
+  return static_cast<unsigned>(g);
+}
+
+cudaError_t launch_project_planes(int fmt, const PlaneTable &t, int64_t *acc, cudaStream_t stream) {
+  const unsigned grid = planes_grid(t);
+  if (grid == 0) {  // no blocks at all: the counters still receive 0
+    for (int j = 0; j < t.n; ++j)
+      if (t.p[j].counter) {
+        cudaError_t e = cudaMemsetAsync(t.p[j].counter, 0, sizeof(int32_t), stream);
+        if (e != cudaSuccess) return e;
+      }
+    return cudaSuccess;
+  }
+  if (fmt == 0)
+    sq_project_planes_kernel<0><<<grid, kThreads, 0, stream>>>(t, acc);
+  else
+    sq_project_planes_kernel<1><<<grid, kThreads, 0, stream>>>(t, acc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_planes(int fmt, const PlaneTable &t, int64_t *acc, cudaStream_t stream) {
+  const unsigned grid = planes_grid(t);
+  if (grid == 0) {
+    for (int j = 0; j < t.n; ++j)
+      if (t.p[j].counter) {
+        cudaError_t e = cudaMemsetAsync(t.p[j].counter, 0, sizeof(int64_t), stream);
+        if (e != cudaSuccess) return e;
+      }
+    return cudaSuccess;
+  }
+  if (fmt == 0)
+    sq_merge_planes_kernel<0><<<grid, kThreads, 0, stream>>>(t, acc);
+  else
+    sq_merge_planes_kernel<1><<<grid, kThreads, 0, stream>>>(t, acc);
   return cudaGetLastError();
 }
 

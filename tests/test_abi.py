@@ -183,3 +183,31 @@ def test_variant_validation(built):
     ok = L._SqControlWeight(8, 64, A16, A16)
     assert h.status_of("sq_control_fwd", ctypes.byref(ok), None, 0, None, None) == 0
     assert h.status_of("sq_lowrank_product", 8, 8, 300, 1.0, vp(A16), vp(A16), vp(A16), None) == -1   # r > 256
+
+
+def test_plane_table_validation(built):
+    """The multi-plane projection and merge check every plane (count, shape,
+    alignment, ws2) before anything is launched; zero planes is a no-op."""
+    h = pkg.Handle()
+    P = pkg._lib._SqPlane
+
+    def call(name, planes, n=None, fmt=0):
+        arr = (P * max(1, len(planes)))(*planes)
+        return h.status_of(name, fmt, len(planes) if n is None else n, arr, None)
+
+    ok = P(8, 16, 0.5, A16, A16, A16, A16, A16, A16)
+    for name in ("sq_project_planes", "sq_merge_planes"):
+        assert call(name, []) == 0
+        assert call(name, [ok], n=17) == -1 and "nplanes" in h.last_error()
+        assert call(name, [ok], n=-1) == -1
+        assert h.status_of(name, 0, 2, None, None) == -1
+        assert call(name, [ok, P(8, 16, 0.0, A16, A16, None, None, None, None)]) == -1 and "ws2" in h.last_error()
+        assert call(name, [P(8, 16, 2.0, A16, A16, None, None, None, None)], fmt=1) == -1
+        assert call(name, [P(-8, 16, 1.0, A16, A16, None, None, None, None)]) == -1
+        assert call(name, [P(1, 8, 1.0, A16, A16, None, None, None, None)]) == -1 and "multiple of 16" in h.last_error()
+        assert call(name, [P(8, 16, 1.0, 0, A16, None, None, None, None)]) == -1 and "latent" in h.last_error()
+        assert call(name, [P(8, 16, 1.0, A16, A16 + 4, None, None, None, None)]) == -1
+    assert call("sq_project_planes", [P(8, 16, 1.0, A16, A16, A16 + 8, None, None, None)]) == -1
+    assert call("sq_project_planes", [P(8, 16, 1.0, A16, A16, None, None, A16 + 2, None)]) == -1
+    assert call("sq_merge_planes", [P(8, 16, 1.0, A16, A16, None, A16 + 8, None, None)]) == -1
+    assert call("sq_merge_planes", [P(8, 16, 1.0, A16, A16, None, None, None, A16 + 4)]) == -1

@@ -228,6 +228,85 @@ def test_layer_merge_c5(h):
     assert 0.005 < frac < 0.2, frac
 
 
+def test_layer_planes_in_one_launch_c5(h):
+    """The 7 scale planes of the layer projected in one launch and merged in one
+    launch (sq_project_planes / sq_merge_planes): bytes, masks, NaN counts, merged
+    planes, on-grid deltas and changed counts bit-exact against the oracle, twice in
+    a row (the counters' accumulators reset between calls)."""
+    from paper_2609_04526_gb300 import synth
+    wl = synth.WORKLOADS["c5"]
+    st = []
+    for lin in wl.linears:
+        w = synth.gen_weight(wl, lin, device="cuda")
+        L = synth.gen_latent(wl, lin, w, device="cuda")
+        L[5, :3] = float("nan")
+        st.append(dict(w=w, L=L, b=torch.empty_like(w.scales), m=torch.empty_like(w.scales),
+                       nf=torch.full((1,), -3, dtype=torch.int32, device="cuda"), art=w.scales.clone(),
+                       d=torch.empty_like(L), ch=torch.full((1,), -3, dtype=torch.int64, device="cuda")))
+    for rep in range(2):
+        h.sq_project_planes(wl.fmt, [dict(latent=x["L"], bytes=x["b"], mask=x["m"], nonfinite=x["nf"], ws2=x["w"].ws2)
+                                     for x in st])
+        olds = [x["art"].clone() for x in st]
+        h.sq_merge_planes(wl.fmt, [dict(latent=x["L"], bytes=x["art"], ongrid_delta=x["d"], changed=x["ch"],
+                                        ws2=x["w"].ws2) for x in st])
+        h.sq_sync()
+        for x, old in zip(st, olds):
+            Lh = host(x["L"])
+            rb, rm, rnf = oracle.project(wl.fmt, Lh, x["w"].ws2)
+            assert np.array_equal(host(x["b"]), rb) and np.array_equal(host(x["m"]), rm)
+            assert int(x["nf"].item()) == rnf == 3
+            rs, rd, rch = oracle.merge(wl.fmt, Lh, host(old), x["w"].ws2)
+            assert np.array_equal(host(x["art"]), rs) and int(x["ch"].item()) == rch
+            assert rch > 0 if rep == 0 else rch == 0
+            dh = host(x["d"])
+            assert np.array_equal(np.isnan(dh), np.isnan(rd))
+            assert np.array_equal(dh.view(np.uint32)[~np.isnan(dh)], rd.view(np.uint32)[~np.isnan(rd)])
+
+
+@pytest.mark.parametrize("fmt", [NV, MX])
+def test_planes_of_mixed_shapes(h, fmt):
+    """16 planes of different shapes (one block row up to a few thousand rows, the
+    CTA boundaries of the one-launch kernel falling inside and between planes), edge
+    latents and NaNs, per-plane ws2: equal to the oracle and to one single-plane
+    call per plane, counters per plane."""
+    rng = np.random.default_rng(41 + fmt)
+    shapes = [(8, 16), (1, 16), (24, 32), (640, 48), (3, 256), (1000, 16), (16, 16), (2048, 64), (5, 32), (8, 896),
+              (100, 160), (1, 32), (64, 16), (4096, 16), (7, 48), (33, 16)]
+    planes, singles = [], []
+    for j, (N, G) in enumerate(shapes):
+        ws2 = float(np.float32(2.0 ** rng.integers(-12, 2) * rng.uniform(1, 2))) if fmt == NV else 1.0
+        base = 448.0 * ws2 if fmt == NV else 1.0
+        L = (rng.standard_normal((N, G)) * base * (0.3 if fmt == NV else 4.0)).astype(np.float32)
+        if fmt == MX:
+            L = np.exp2(L).astype(np.float32)
+        L.flat[rng.integers(0, L.size, 1 + j % 3)] = np.nan
+        L.flat[0] = base * 3
+        Ld = torch.from_numpy(L).cuda()
+        art = torch.from_numpy(rng.integers(0, 0x7F if fmt == NV else 255, size=(N, G), dtype=np.uint8)).cuda()
+        planes.append(dict(latent=Ld, bytes=torch.empty(N, G, dtype=torch.uint8, device="cuda"),
+                           mask=torch.empty(N, G, dtype=torch.uint8, device="cuda"),
+                           nonfinite=torch.full((1,), 9, dtype=torch.int32, device="cuda"), ws2=ws2,
+                           art=art, art0=art.clone(), ongrid_delta=torch.empty_like(Ld),
+                           changed=torch.full((1,), 9, dtype=torch.int64, device="cuda")))
+    h.sq_project_planes(fmt, planes)
+    h.sq_merge_planes(fmt, [dict(latent=p["latent"], bytes=p["art"], ongrid_delta=p["ongrid_delta"],
+                                 changed=p["changed"], ws2=p["ws2"]) for p in planes])
+    h.sq_sync()
+    for p in planes:
+        Lh = host(p["latent"])
+        rb, rm, rnf = oracle.project(fmt, Lh, p["ws2"])
+        assert np.array_equal(host(p["bytes"]), rb) and np.array_equal(host(p["mask"]), rm)
+        assert int(p["nonfinite"].item()) == rnf
+        rs, rd, rch = oracle.merge(fmt, Lh, host(p["art0"]), p["ws2"])
+        assert np.array_equal(host(p["art"]), rs) and int(p["changed"].item()) == rch
+        dh = host(p["ongrid_delta"])
+        assert np.array_equal(np.isnan(dh), np.isnan(rd))
+        assert np.array_equal(dh.view(np.uint32)[~np.isnan(dh)], rd.view(np.uint32)[~np.isnan(rd)])
+        b1, m1 = h.sq_project_scales(fmt, p["latent"], p["ws2"])
+        h.sq_sync()
+        assert torch.equal(b1, p["bytes"]) and torch.equal(m1, p["mask"])
+
+
 @pytest.mark.parametrize("key,fmt,M,N,K", [SMALL[0], SMALL[2]], ids=["c1", "mx_ragged"])
 def test_merged_artifact_is_the_trained_weight(h, key, fmt, M, N, K):
     """max|dW| = 0 in weight space (Sec. 3, merge): the artifact (unchanged codes plus the
