@@ -16,7 +16,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libscaleqlora.so")
-SOURCES = ["sq_api.cu", "sq_gemm.cu", "sq_grouped.cu", "sq_control.cu", "sq_project.cu", "sq_noalloc.cu"]
+SOURCES = ["sq_api.cu", "sq_gemm.cu", "sq_grouped.cu", "sq_control.cu", "sq_project.cu", "sq_noalloc.cu",
+           "sq_adapter_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", f"-I{INCLUDE}", f"-I{CSRC}"]
 

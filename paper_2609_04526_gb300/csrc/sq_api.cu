@@ -937,7 +937,7 @@ sq_status sq_lowrank_grad(sq_handle h, int64_t N, int64_t G, int32_t r, float al
   SQ_TRY(check_buf(h, A, "A"));
   SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count), st));
   e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace.ptr),
-                               dev->sm_count, st);
+                               dev->sm_count, st, dev->err_word);
   if (e != cudaSuccess) return cuda_fail(h, e, "adapter gradient launch");
   return SQ_OK;
   SQ_GUARD_END
@@ -1219,7 +1219,7 @@ sq_status sq_grouped_lowrank_grad(sq_handle h, int32_t E, int64_t N, int64_t G, 
   SQ_TRY(check_buf(h, A, "A"));
   SQ_TRY(ensure_workspace(h, dev, sqi::lowrank_grad_workspace(N, G, r, dev->sm_count, E), st));
   e = sqi::launch_lowrank_grad(N, G, r, alpha_over_r, g, B, A, dB, dA, static_cast<float *>(dev->workspace.ptr),
-                               dev->sm_count, st, E);
+                               dev->sm_count, st, dev->err_word, E);
   if (e != cudaSuccess) return cuda_fail(h, e, "grouped adapter gradient launch");
   return SQ_OK;
   SQ_GUARD_END

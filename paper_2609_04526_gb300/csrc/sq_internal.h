@@ -170,10 +170,17 @@ cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float w
                                    const uint8_t *base, const uint16_t *B, const uint16_t *A, uint8_t *bytes_out,
                                    uint8_t *mask_out, int32_t *nonfinite, float *latent_out, cudaStream_t stream,
                                    int experts = 1, const float *ws2_per = nullptr);
+// Ranks up to 128 run on the tensor cores (sq_adapter_tc.cu), larger ones on CUDA
+// cores; `err` is the device error word (bounded waits of the tensor-core path).
 size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count, int experts = 1);
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
-                                cudaStream_t stream, int experts = 1);
+                                cudaStream_t stream, int *err, int experts = 1);
+bool lowrank_grad_tc_supported(int r);
+size_t lowrank_grad_tc_workspace(int64_t N, int64_t G, int r, int experts, int sm_count);
+cudaError_t launch_lowrank_grad_tc(int64_t N, int64_t G, int r, float alpha_over_r, const float *g,
+                                   const uint16_t *B, const uint16_t *A, float *dB, float *dA, float *workspace,
+                                   int *err, int sm_count, cudaStream_t stream, int experts);
 constexpr int kMaxLowRank = 256;  // r limit of the adapter kernels
 
 // Scale-family variants (ablation appendix): the least-squares code-preserving fit

@@ -290,9 +290,13 @@ __device__ __forceinline__ void plane_counters(const PlaneTable &t, int j, uint3
   *ticket = 0u;
 }
 
+// A thread loads all its vectors' latents (and, merging, the old bytes) before it
+// computes and stores any: the byte stores could alias the latent loads as far as
+// the compiler knows, so interleaving them would serialise every vector on the
+// memory latency.
 template <int FMT>
-__global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
-                                                                     int64_t *acc) {
+__global__ void __launch_bounds__(kThreads, 2) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
+                                                                        int64_t *acc) {
   __shared__ uint32_t red[kThreads / 32];
   int64_t first_block;
   const int j = plane_of_block(t, blockIdx.x, first_block);
@@ -300,26 +304,32 @@ __global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __gri
   const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;  // the same IEEE fp32 product as the single-plane cap
   const int64_t nvec = pl.count / 16;
   const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
+  float L[kPlaneVecsPerThread][16];
+#pragma unroll
+  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
+    const int64_t v = v0 + r * kThreads;
+    if (v < nvec) {
+      const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float4 f = __ldcs(src + q);
+        L[r][4 * q] = f.x;
+        L[r][4 * q + 1] = f.y;
+        L[r][4 * q + 2] = f.z;
+        L[r][4 * q + 3] = f.w;
+      }
+    }
+  }
   uint32_t nan_count = 0;
 #pragma unroll
   for (int r = 0; r < kPlaneVecsPerThread; ++r) {
     const int64_t v = v0 + r * kThreads;
     if (v >= nvec) break;
-    const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
-    float L[16];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 f = __ldcs(src + q);
-      L[4 * q] = f.x;
-      L[4 * q + 1] = f.y;
-      L[4 * q + 2] = f.z;
-      L[4 * q + 3] = f.w;
-    }
     uint32_t ob[4] = {0, 0, 0, 0}, om[4] = {0, 0, 0, 0};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       uint32_t b, m, n;
-      project_one<FMT>(L[i], ws2, cap, b, m, n);
+      project_one<FMT>(L[r][i], ws2, cap, b, m, n);
       ob[i >> 2] |= b << (8 * (i & 3));
       om[i >> 2] |= m << (8 * (i & 3));
       nan_count += n;
@@ -331,8 +341,8 @@ __global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __gri
 }
 
 template <int FMT>
-__global__ void __launch_bounds__(kThreads) sq_merge_planes_kernel(const __grid_constant__ PlaneTable t,
-                                                                   int64_t *acc) {
+__global__ void __launch_bounds__(kThreads, 2) sq_merge_planes_kernel(const __grid_constant__ PlaneTable t,
+                                                                      int64_t *acc) {
   __shared__ uint32_t red[kThreads / 32];
   int64_t first_block;
   const int j = plane_of_block(t, blockIdx.x, first_block);
@@ -340,29 +350,36 @@ __global__ void __launch_bounds__(kThreads) sq_merge_planes_kernel(const __grid_
   const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;
   const int64_t nvec = pl.count / 16;
   const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
+  float L[kPlaneVecsPerThread][16];
+  uint4 old4[kPlaneVecsPerThread];
+#pragma unroll
+  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
+    const int64_t v = v0 + r * kThreads;
+    if (v < nvec) {
+      const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float4 f = __ldcs(src + q);
+        L[r][4 * q] = f.x;
+        L[r][4 * q + 1] = f.y;
+        L[r][4 * q + 2] = f.z;
+        L[r][4 * q + 3] = f.w;
+      }
+      old4[r] = *(reinterpret_cast<const uint4 *>(pl.bytes) + v);
+    }
+  }
   uint32_t n_changed = 0;
 #pragma unroll
   for (int r = 0; r < kPlaneVecsPerThread; ++r) {
     const int64_t v = v0 + r * kThreads;
     if (v >= nvec) break;
-    const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
-    float L[16];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 f = __ldcs(src + q);
-      L[4 * q] = f.x;
-      L[4 * q + 1] = f.y;
-      L[4 * q + 2] = f.z;
-      L[4 * q + 3] = f.w;
-    }
-    const uint4 old4 = *(reinterpret_cast<const uint4 *>(pl.bytes) + v);
-    const uint32_t old[4] = {old4.x, old4.y, old4.z, old4.w};
+    const uint32_t old[4] = {old4[r].x, old4[r].y, old4[r].z, old4[r].w};
     uint32_t ob[4] = {0, 0, 0, 0};
     float d[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       uint32_t b, m, n;
-      project_one<FMT>(L[i], ws2, cap, b, m, n);
+      project_one<FMT>(L[r][i], ws2, cap, b, m, n);
       const uint32_t o = (old[i >> 2] >> (8 * (i & 3))) & 0xFFu;
       ob[i >> 2] |= b << (8 * (i & 3));
       n_changed += (b != o) ? 1u : 0u;
@@ -1028,6 +1045,7 @@ cudaError_t launch_project_lowrank(int fmt, int64_t N, int64_t G, int r, float w
 
 // Workspace of the adapter gradients: the partial products of dB and of dA (all experts).
 size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count, int experts) {
+  if (lowrank_grad_tc_supported(r)) return lowrank_grad_tc_workspace(N, G, r, experts, sm_count);
   const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT) * experts;
   const int64_t ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT) * experts;
   const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);
@@ -1036,7 +1054,9 @@ size_t lowrank_grad_workspace(int64_t N, int64_t G, int r, int sm_count, int exp
 
 cudaError_t launch_lowrank_grad(int64_t N, int64_t G, int r, float alpha_over_r, const float *g, const uint16_t *B,
                                 const uint16_t *A, float *dB, float *dA, float *workspace, int sm_count,
-                                cudaStream_t stream, int experts) {
+                                cudaStream_t stream, int *err, int experts) {
+  if (lowrank_grad_tc_supported(r))
+    return launch_lowrank_grad_tc(N, G, r, alpha_over_r, g, B, A, dB, dA, workspace, err, sm_count, stream, experts);
   const int64_t tb = ((N + kT - 1) / kT) * ((r + kT - 1) / kT) * experts;
   const int64_t ta = ((r + kT - 1) / kT) * ((G + kT - 1) / kT) * experts;
   const int64_t cb = adapter_chunks(G, tb, sm_count), ca = adapter_chunks(N, ta, sm_count);

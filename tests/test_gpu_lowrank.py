@@ -78,7 +78,8 @@ def test_adapter_projection_bit_exact(h, key, fmt, N, G, r):
     _check_projection(h, fmt, w.scales, B, A, w.ws2, aor)
 
 
-@pytest.mark.parametrize("N,G,r", [(1, 16, 1), (40, 48, 13), (300, 96, 58), (1000, 32, 256), (129, 1040, 7)])
+@pytest.mark.parametrize("N,G,r", [(1, 16, 1), (40, 48, 13), (300, 96, 58), (1000, 32, 256), (129, 1040, 7),
+                                   (256, 64, 128), (64, 32, 129)])
 def test_adapter_gradients_match_oracle_and_repeat(h, N, G, r):
     gen = torch.Generator(device="cuda").manual_seed(N * 131 + G * 7 + r)
     g = torch.randn(N, G, device="cuda", generator=gen)
