@@ -238,7 +238,7 @@ __global__ void __launch_bounds__(kThreads) sq_merge_kernel(int64_t count, float
 // plane j - 1), so it reduces its counter within the block and adds it with one
 // atomic; the last CTA to finish (a ticket) writes every plane's count and clears
 // the accumulators for the next call.
-constexpr int kPlaneVecsPerThread = 4;
+constexpr int kPlaneVecsPerThread = 2;
 constexpr int kPlaneVecs = kThreads * kPlaneVecsPerThread;
 
 __device__ __forceinline__ int plane_of_block(const PlaneTable &t, int64_t b, int64_t &first_block) {
@@ -295,7 +295,7 @@ __device__ __forceinline__ void plane_counters(const PlaneTable &t, int j, uint3
 // the compiler knows, so interleaving them would serialise every vector on the
 // memory latency.
 template <int FMT>
-__global__ void __launch_bounds__(kThreads, 2) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
+__global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
                                                                         int64_t *acc) {
   __shared__ uint32_t red[kThreads / 32];
   int64_t first_block;
@@ -341,7 +341,7 @@ __global__ void __launch_bounds__(kThreads, 2) sq_project_planes_kernel(const __
 }
 
 template <int FMT>
-__global__ void __launch_bounds__(kThreads, 2) sq_merge_planes_kernel(const __grid_constant__ PlaneTable t,
+__global__ void __launch_bounds__(kThreads) sq_merge_planes_kernel(const __grid_constant__ PlaneTable t,
                                                                       int64_t *acc) {
   __shared__ uint32_t red[kThreads / 32];
   int64_t first_block;
