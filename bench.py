@@ -984,7 +984,8 @@ class MoEState:
         self.counts = synth.gen_routing(wl)
         self.off = synth.offsets_of(self.counts)
         M = self.off[-1]
-        self.acts = {name: synth.gen_act(wl, name, M=M, device=device) for name, _, _ in wl.acts}
+        self.acts = {name: synth.gen_act(wl, name, M=M, device=device) for name, _, _ in wl.acts
+                     if any(l.x == name for l in wl.linears)}
         self.lin = []
         for lin in wl.linears:
             ex = synth.gen_experts(wl, lin, device=device)
@@ -1143,6 +1144,13 @@ def run_moe(args):
     torch.cuda.set_device(local)
     build.build()
     wl = synth.MOE_WORKLOADS[args.moe]
+    if args.linears:
+        import dataclasses
+        keep = args.linears.split(",")
+        wl = dataclasses.replace(wl, linears=tuple(l for l in wl.linears if l.name in keep),
+                                 title=f"{wl.title}, only {args.linears}")
+        if not wl.linears:
+            raise SystemExit(f"--linears {args.linears}: no such linear in {args.moe}")
     pk = peaks()
     h = pkg.Handle()
     stream = torch.cuda.current_stream()
