@@ -39,6 +39,9 @@ KINDS_LOWRANK = ("project", "fwd", "dx", "sgrad", "adapter_grad", "merge")
 # GB300 datasheet figures (dense, no sparsity): the fractions against these sit beside
 # the ones against the measured torch matmul / copy rates.
 DATASHEET = {"bf16_tflops": 2250.0, "hbm_gbs": 7900.0}
+# The tensor pipe's dense bf16 rate per GHz of SM clock: 4096 multiply-adds per SM per
+# cycle (measured with tcgen05 MMAs on static operands) on 152 SMs.
+TENSOR_TFLOPS_PER_GHZ = 2 * 4096 * 152 / 1e3
 ADAPTER_RANK = 58  # the paper's Llama-3-8B scale rank (Sec. 5 recipe)
 
 
@@ -238,7 +241,8 @@ class ClockSampler:
 
 def per_ghz(kernels, clk):
     """Clock-normalised figures of each kernel kind: throughput per GHz of the median
-    sampled SM clock, and the step's share of that kind in millions of SM cycles."""
+    sampled SM clock, the step's share of that kind in millions of SM cycles, and for
+    contractions the fraction of the tensor pipe's peak at that clock."""
     if not clk or not clk.get("sm_mhz"):
         return
     ghz = clk["sm_mhz"] / 1e3
@@ -246,6 +250,8 @@ def per_ghz(kernels, clk):
         k["per_ghz"] = k["achieved"] / ghz
         k["per_ghz_unit"] = k["unit"] + " per GHz"
         k["mcycles_per_step"] = k["ms_per_step"] * clk["sm_mhz"] / 1e3
+        if k["unit"] == "TFLOP/s":
+            k["frac_of_tensor_pipe_at_sampled_clock"] = k["per_ghz"] / TENSOR_TFLOPS_PER_GHZ
 
 
 # --------------------------------------------------------------------- workload
@@ -952,7 +958,10 @@ def run_ours(args):
                          "traffic_note": "ncu dram bytes per launch, mean over the layer's 7 launches of this kernel "
                                          "(profiles/traffic_c5_layer_step.json); null if its sources changed since",
                          "peak_source": f"{pk['source']} bf16 sustained (torch.matmul 8192^3 held for 4 s)",
-                         "frac_vs_datasheet": k["achieved"] / DATASHEET["bf16_tflops"]},
+                         "frac_vs_datasheet": k["achieved"] / DATASHEET["bf16_tflops"],
+                         "frac_of_tensor_pipe_at_sampled_clock": k.get("frac_of_tensor_pipe_at_sampled_clock"),
+                         "tensor_pipe_peak_at_sampled_clock": (TENSOR_TFLOPS_PER_GHZ * clk["sm_mhz"] / 1e3
+                                                               if clk and clk.get("sm_mhz") else None)},
             "fraction_of_peak": {"bf16_burst_measured_matmul": value / world / pk["bf16"],
                                  "bf16_sustained_measured_matmul": value / world / pk["bf16_sustained"],
                                  "bf16_datasheet_dense": value / world / DATASHEET["bf16_tflops"]},
