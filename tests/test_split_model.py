@@ -1,9 +1,10 @@
 """The token-split rule of the dense scale gradient (host logic, no GPU).
 
 sgrad_splits(tiles, clusters, M) in csrc/sq_internal.h picks how many token parts a
-dense scale-gradient launch uses: the part count s <= 8 (each part >= 2048 tokens) that
-minimises ceil(tiles * s / clusters) / s + 0.01 (s - 1), the launch's length in units of
-one full-M tile per cluster plus a small charge per extra part. Checked here by compiling
+dense scale-gradient launch uses: with w(s) = ceil(tiles * s / clusters) / s, the launch's
+length in units of one full-M tile per cluster, the largest part count s <= 8 (each part
+>= 2048 tokens) whose w(s) is within 1 % of the smallest and no longer than w(1): more,
+shorter parts keep the dY and X panels that a part's waves share in L2. Checked here by compiling
 the header's inline function into a tiny host program and comparing it with the same
 rule evaluated in Python, and on the shapes it is meant for.
 """
@@ -31,14 +32,10 @@ int main() {
 
 
 def _rule(tiles, clusters, M):
-    best, best_cost = 1, float(math.ceil(tiles / clusters))
-    for s in range(2, 9):
-        if M < s * 2048:
-            break
-        cost = math.ceil(tiles * s / clusters) / s + 0.01 * (s - 1)
-        if cost < best_cost - 1e-9:
-            best, best_cost = s, cost
-    return best
+    top = max(1, min(8, M // 2048))
+    w = {s: math.ceil(tiles * s / clusters) / s for s in range(1, top + 1)}
+    limit = min(min(w.values()) * 1.01, w[1])
+    return max(s for s in w if w[s] <= limit + 1e-9)
 
 
 @pytest.fixture(scope="module")
@@ -67,7 +64,7 @@ def test_layer_shapes(splits):
     M, C = 32768, 76
     shapes = {"q/o": (4096, 4096), "k/v": (1024, 4096), "gate/up": (14336, 4096), "down": (4096, 14336)}
     got = splits([(tiles_of(N, K), C, M) for N, K in shapes.values()])
-    assert got == [5, 7, 5, 5]
+    assert got == [8, 7, 8, 8]
 
 
 def test_few_tokens_never_split(splits):
