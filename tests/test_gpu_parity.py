@@ -504,6 +504,34 @@ def test_projection_dense_sweep_bit_exact(h):
     assert np.array_equal(host(b), rb) and np.array_equal(host(m), rm)
 
 
+@pytest.mark.parametrize("ws2", [0.00731, 1.0, 0.0123, 2.0 ** -9, 3.3e-4, 5.1e3])
+def test_projection_near_e4m3_midpoints_bit_exact(h, ws2):
+    """Latents whose quotient by ws2 lies at, or within 40 fp32 ulps of, every
+    rounding midpoint and grid value of E4M3 (normal and subnormal range, both
+    signs), each also nudged by one ulp of the latent: the projected bytes and mask
+    equal the oracle's. These are the values where rounding the quotient to E4M3
+    depends on its last bits."""
+    ws2 = float(np.float32(ws2))
+    grid = np.array([m * 2.0 ** -9 for m in range(1, 8)] +
+                    [(1 + m / 8) * 2.0 ** e for e in range(-6, 9) for m in range(8)], dtype=np.float64)
+    grid = grid[grid <= 448]
+    mids = (grid[:-1] + grid[1:]) / 2
+    t = np.concatenate([grid, mids, [2.0 ** -10]]).astype(np.float32)
+    k = np.arange(-40, 41, dtype=np.int64)
+    tb = (t.view(np.uint32).astype(np.int64)[:, None] + k[None, :]).ravel()
+    q = tb[(tb > 0) & (tb < 0x7F800000)].astype(np.uint32).view(np.float32)
+    L = (q.astype(np.float64) * ws2).astype(np.float32)
+    L = np.concatenate([L, np.nextafter(L, np.float32(np.inf)), np.nextafter(L, np.float32(0))])
+    L = np.concatenate([L, -L]).astype(np.float32)
+    L = L[: L.size // 16 * 16].reshape(16, -1)
+    b, m = h.sq_project_scales(NV, torch.from_numpy(L.copy()).cuda(), ws2)
+    h.sq_sync()
+    rb, rm, _ = oracle.project(NV, L, ws2)
+    bad = np.nonzero(host(b) != rb)
+    assert np.array_equal(host(b), rb), (L[bad][:8], host(b)[bad][:8], rb[bad][:8])
+    assert np.array_equal(host(m), rm)
+
+
 def test_empty_batch_and_sync(h):
     from paper_2609_04526_gb300 import synth
     wl = synth.custom("e", NV, 4, 64, 128, seed=1)
