@@ -290,10 +290,48 @@ __device__ __forceinline__ void plane_counters(const PlaneTable &t, int j, uint3
   *ticket = 0u;
 }
 
-// A thread loads all its vectors' latents (and, merging, the old bytes) before it
-// computes and stores any: the byte stores could alias the latent loads as far as
-// the compiler knows, so interleaving them would serialise every vector on the
-// memory latency.
+// Four consecutive blocks of a plane (one float4 of latents) -> their bytes, mask bytes
+// and NaN count, each block exactly as project_one. NVFP4 converts two blocks per
+// instruction; a NaN latent's byte is patched afterwards (rare).
+template <int FMT>
+__device__ __forceinline__ void project4(float4 L4, float ws2, float cap, uint32_t &bytes, uint32_t &mask,
+                                         uint32_t &nan) {
+  const float l[4] = {L4.x, L4.y, L4.z, L4.w};
+  bytes = mask = nan = 0;
+  if (FMT == 0) {
+    float q[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      nan += (l[c] != l[c]) ? 1u : 0u;
+      mask |= (fabsf(l[c]) <= cap ? 1u : 0u) << (8 * c);  // false for NaN, as -cap <= L <= cap
+      q[c] = __fdiv_rn(fminf(fmaxf(l[c], -cap), cap), ws2);
+    }
+    bytes = e4m3x2_rn(q[0], q[1]) | (e4m3x2_rn(q[2], q[3]) << 16);
+    if (nan) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        if (l[c] != l[c]) bytes = (bytes & ~(0xFFu << (8 * c))) | (0x7Fu << (8 * c));
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      uint32_t b, m, n;
+      project_one<FMT>(l[c], ws2, cap, b, m, n);
+      bytes |= b << (8 * c);
+      mask |= m << (8 * c);
+      nan += n;
+    }
+  }
+}
+
+// A CTA's chunk is kPlaneVecs x 16 blocks: lane t of the CTA takes float4 t + kThreads * i
+// of it (i < 4 kPlaneVecsPerThread), so each warp-wide load reads 512 contiguous bytes and
+// each store of bytes writes 128. A thread loads all its latents (and, merging, the old
+// bytes) before it computes and stores any: the byte stores could alias the latent
+// loads as far as the compiler knows, so interleaving them would serialise every
+// float4 on the memory latency.
+constexpr int kPlaneF4 = 4 * kPlaneVecsPerThread;  // float4s per thread per chunk
+
 template <int FMT>
 __global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __grid_constant__ PlaneTable t,
                                                                         int64_t *acc) {
@@ -302,40 +340,25 @@ __global__ void __launch_bounds__(kThreads) sq_project_planes_kernel(const __gri
   const int j = plane_of_block(t, blockIdx.x, first_block);
   const PlaneArgs &pl = t.p[j];
   const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;  // the same IEEE fp32 product as the single-plane cap
-  const int64_t nvec = pl.count / 16;
-  const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
-  float L[kPlaneVecsPerThread][16];
+  const int64_t nf4 = pl.count / 4;
+  const int64_t f0 = (static_cast<int64_t>(blockIdx.x) - first_block) * (4 * kPlaneVecs) + threadIdx.x;
+  const float4 *src = reinterpret_cast<const float4 *>(pl.latent);
+  float4 L[kPlaneF4];
 #pragma unroll
-  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
-    const int64_t v = v0 + r * kThreads;
-    if (v < nvec) {
-      const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float4 f = __ldcs(src + q);
-        L[r][4 * q] = f.x;
-        L[r][4 * q + 1] = f.y;
-        L[r][4 * q + 2] = f.z;
-        L[r][4 * q + 3] = f.w;
-      }
-    }
+  for (int i = 0; i < kPlaneF4; ++i) {
+    const int64_t f = f0 + static_cast<int64_t>(i) * kThreads;
+    if (f < nf4) L[i] = __ldcs(src + f);
   }
   uint32_t nan_count = 0;
 #pragma unroll
-  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
-    const int64_t v = v0 + r * kThreads;
-    if (v >= nvec) break;
-    uint32_t ob[4] = {0, 0, 0, 0}, om[4] = {0, 0, 0, 0};
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      uint32_t b, m, n;
-      project_one<FMT>(L[r][i], ws2, cap, b, m, n);
-      ob[i >> 2] |= b << (8 * (i & 3));
-      om[i >> 2] |= m << (8 * (i & 3));
-      nan_count += n;
-    }
-    __stcs(reinterpret_cast<uint4 *>(pl.bytes) + v, make_uint4(ob[0], ob[1], ob[2], ob[3]));
-    if (pl.mask) __stcs(reinterpret_cast<uint4 *>(pl.mask) + v, make_uint4(om[0], om[1], om[2], om[3]));
+  for (int i = 0; i < kPlaneF4; ++i) {
+    const int64_t f = f0 + static_cast<int64_t>(i) * kThreads;
+    if (f >= nf4) break;
+    uint32_t by, mk, na;
+    project4<FMT>(L[i], ws2, cap, by, mk, na);
+    __stcs(reinterpret_cast<unsigned int *>(pl.bytes) + f, by);
+    if (pl.mask) __stcs(reinterpret_cast<unsigned int *>(pl.mask) + f, mk);
+    nan_count += na;
   }
   plane_counters<false>(t, j, nan_count, acc, red);
 }
@@ -348,48 +371,35 @@ __global__ void __launch_bounds__(kThreads) sq_merge_planes_kernel(const __grid_
   const int j = plane_of_block(t, blockIdx.x, first_block);
   const PlaneArgs &pl = t.p[j];
   const float ws2 = pl.ws2, cap = 448.0f * pl.ws2;
-  const int64_t nvec = pl.count / 16;
-  const int64_t v0 = (static_cast<int64_t>(blockIdx.x) - first_block) * kPlaneVecs + threadIdx.x;
-  float L[kPlaneVecsPerThread][16];
-  uint4 old4[kPlaneVecsPerThread];
+  const int64_t nf4 = pl.count / 4;
+  const int64_t f0 = (static_cast<int64_t>(blockIdx.x) - first_block) * (4 * kPlaneVecs) + threadIdx.x;
+  const float4 *src = reinterpret_cast<const float4 *>(pl.latent);
+  uint32_t *art = reinterpret_cast<uint32_t *>(pl.bytes);
+  float4 L[kPlaneF4];
+  uint32_t old[kPlaneF4];
 #pragma unroll
-  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
-    const int64_t v = v0 + r * kThreads;
-    if (v < nvec) {
-      const float4 *src = reinterpret_cast<const float4 *>(pl.latent) + 4 * v;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float4 f = __ldcs(src + q);
-        L[r][4 * q] = f.x;
-        L[r][4 * q + 1] = f.y;
-        L[r][4 * q + 2] = f.z;
-        L[r][4 * q + 3] = f.w;
-      }
-      old4[r] = *(reinterpret_cast<const uint4 *>(pl.bytes) + v);
+  for (int i = 0; i < kPlaneF4; ++i) {
+    const int64_t f = f0 + static_cast<int64_t>(i) * kThreads;
+    if (f < nf4) {
+      L[i] = __ldcs(src + f);
+      old[i] = art[f];
     }
   }
   uint32_t n_changed = 0;
 #pragma unroll
-  for (int r = 0; r < kPlaneVecsPerThread; ++r) {
-    const int64_t v = v0 + r * kThreads;
-    if (v >= nvec) break;
-    const uint32_t old[4] = {old4[r].x, old4[r].y, old4[r].z, old4[r].w};
-    uint32_t ob[4] = {0, 0, 0, 0};
-    float d[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      uint32_t b, m, n;
-      project_one<FMT>(L[r][i], ws2, cap, b, m, n);
-      const uint32_t o = (old[i >> 2] >> (8 * (i & 3))) & 0xFFu;
-      ob[i >> 2] |= b << (8 * (i & 3));
-      n_changed += (b != o) ? 1u : 0u;
-      d[i] = __fsub_rn(scale_value<FMT>(b, ws2), scale_value<FMT>(o, ws2));
-    }
-    *(reinterpret_cast<uint4 *>(pl.bytes) + v) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+  for (int i = 0; i < kPlaneF4; ++i) {
+    const int64_t f = f0 + static_cast<int64_t>(i) * kThreads;
+    if (f >= nf4) break;
+    uint32_t by, mk, na;
+    project4<FMT>(L[i], ws2, cap, by, mk, na);
+    art[f] = by;
+    n_changed += static_cast<uint32_t>(__popc(__vcmpne4(by, old[i]))) >> 3;  // 0xFF per differing byte
     if (pl.delta) {
-      float4 *dst = reinterpret_cast<float4 *>(pl.delta) + 4 * v;
+      float d[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) __stcs(dst + q, make_float4(d[4 * q], d[4 * q + 1], d[4 * q + 2], d[4 * q + 3]));
+      for (int c = 0; c < 4; ++c)
+        d[c] = __fsub_rn(scale_value<FMT>((by >> (8 * c)) & 0xFFu, ws2), scale_value<FMT>((old[i] >> (8 * c)) & 0xFFu, ws2));
+      __stcs(reinterpret_cast<float4 *>(pl.delta) + f, make_float4(d[0], d[1], d[2], d[3]));
     }
   }
   plane_counters<true>(t, j, n_changed, acc, red);
