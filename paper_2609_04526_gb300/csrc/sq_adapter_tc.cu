@@ -99,6 +99,7 @@ __global__ void __launch_bounds__(kAtThreads, 2)
   // One step's gm in registers: thread t covers chunk (t & 7) of rows (t >> 3) + 32 i
   // (8 blocks each), loaded one step ahead of its use.
   const bool vec = (G & 3) == 0;  // rows 16-byte aligned (the plane is)
+  const bool vecA = (G & 7) == 0 && (reinterpret_cast<uintptr_t>(Am) & 15u) == 0;  // A's bf16 rows likewise
   constexpr int kRowsPerThread = kAtRows * 8 / kAtThreads;
   float gv[kRowsPerThread][8];
   auto load = [&](int s) {
@@ -219,15 +220,25 @@ __global__ void __launch_bounds__(kAtThreads, 2)
       st_shared_v4(base + S::kOffG + S::kTile + off, mid[0], mid[1], mid[2], mid[3]);
       st_shared_v4(base + S::kOffG + 2 * S::kTile + off, lo[0], lo[1], lo[2], lo[3]);
     }
-    {  // A's step: rows j < rp16, 8 chunks of 8 blocks; loads first, then the stores
+    {  // A's step: rows j < rp16, 8 chunks of 8 blocks; loads first, then the stores. A chunk
+       // is 16 contiguous bytes of row j: one vector load where rows are 16-byte aligned.
       uint32_t wa[kAtMaxRank * 8 / kAtThreads][4];
 #pragma unroll
       for (int i = 0; i < kAtMaxRank * 8 / kAtThreads; ++i) {
         const int u = threadIdx.x + kAtThreads * i;  // 0 .. 1023 = 128 rows x 8 chunks
         const int j = u >> 3, ch = u & 7;
+        const int64_t bc = b0 + ch * 8;
+        if (vecA && j < r && bc + 8 <= G) {
+          const uint4 a = __ldg(reinterpret_cast<const uint4 *>(Am + j * G + bc));
+          wa[i][0] = a.x;
+          wa[i][1] = a.y;
+          wa[i][2] = a.z;
+          wa[i][3] = a.w;
+          continue;
+        }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const int64_t b = b0 + ch * 8 + 2 * q;
+          const int64_t b = bc + 2 * q;
           const uint32_t lo = (j < r && b < G) ? static_cast<uint32_t>(__ldg(Am + j * G + b)) : 0u;
           const uint32_t hi = (j < r && b + 1 < G) ? static_cast<uint32_t>(__ldg(Am + j * G + b + 1)) : 0u;
           wa[i][q] = lo | (hi << 16);
