@@ -852,8 +852,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       int s = 0, a = 0;             // decoded slot of the current k-step, activation slot of its first half
       uint32_t ph = 0;              // phase parity of the decoded slot
       int tc = 0, it = 0;           // tiles and k-steps of this cluster so far
+      int e_mma = 0;
       bool ok = true;
       for (int tile = cluster; tile < total && ok; tile += nclusters, ++tc) {
+        // A grouped tile whose half 1 lies wholly past its expert's last row skips that
+        // half's MMAs; every wait and commit stays, so the rings keep their phases and
+        // the epilogue (which does not store those rows) still sees accumulator 1 commit.
+        bool skip1 = false;
+        if (GR) {
+          int tm, tn;
+          resolve_tile<GR>(p, tile, e_mma, tm, tn);
+          skip1 = tm * C::kMTile + C::kTile >= group_rows(p, e_mma);
+        }
         for (int kb = 0; kb < num_k; ++kb, ++it) {
           if (!(ok = mbar_spin(&gready[s], ph, abort_flag, p.err))) break;
           const uint64_t b0 = bd_base + static_cast<uint64_t>(s * (C::kB >> 4));
@@ -869,11 +879,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
             if (kb == 0) tc_fence_after();
             const uint32_t d_tmem = tmem_base + h * kTmemCols;
             const uint64_t a0 = ad_base + static_cast<uint64_t>(a * (C::kA >> 4));
+            if (!(h == 1 && skip1)) {
 #pragma unroll
-            for (int kk = 0; kk < C::kBK / 16; ++kk) {
-              const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
-              const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
-              umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+              for (int kk = 0; kk < C::kBK / 16; ++kk) {
+                const uint32_t ka = ((kk >> 2) * 16384 + (kk & 3) * 32) >> 4;
+                const uint32_t kb_ = MODE == MODE_FWD ? ka : (kk * 2048) >> 4;
+                umma_bf16_pair(d_tmem, a0 + ka, b0 + kb_, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+              }
             }
             if (h == 0) umma_commit_pair_mc(&aempty[a]);
             if (kb == num_k - 1) umma_commit_pair_mc(&tfull[h]);  // the epilogue may start on accumulator h
@@ -1127,6 +1139,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
         if (!(ok = mbar_wait(&tfull[h], static_cast<uint32_t>(tc) & 1u, abort_flag, p.err))) break;
         tc_fence_after();
         const int32_t row = tm * C::kMTile + C::kTile * h + 128 * static_cast<int32_t>(rank) + 32 * quad;
+        // a grouped tile's rows past its expert's last row are not stored, so a warp whose
+        // 32 rows all lie there only releases the accumulator (those rows of it may not
+        // even have been computed: see skip1 in the MMA issuer)
+        if (GR && row >= rows) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            if (rank == 0) {
+              if (warp == 0)
+                mbar_arrive_expect_tx(&tempty[h], 4 * C::kEpiWarps);
+              else
+                mbar_arrive(&tempty[h]);
+            } else {
+              st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
+                              mapa_shared(smem_u32(&tempty[h]), 0));
+            }
+          }
+          continue;
+        }
         const uint32_t t_buf = t_row + h * kTmemCols;
         // input gradient and grouped launches: the last 32-column group is read into
         // registers and stored after the accumulator is released
