@@ -72,6 +72,8 @@ SMALL = [
     ("g_mx_many", MX, [0, 0, 0, 5, 130, 0, 512, 513, 1, 0], 40, 96),
     ("g_nv_tail_empty", NV, [77, 0, 0], 8, 32),
     ("g_nv_long_k", NV, [3, 260], 264, 2080),
+    # 256-row tile halves: exactly one half, one row past it, one short of it, a half past a tile
+    ("g_nv_half_edges", NV, [256, 257, 255, 768, 769], 264, 512),
 ]
 
 
