@@ -377,6 +377,9 @@ struct KParams {
 };
 
 // Tuning constants of the decode warps (compile-time; the defaults are the measured best).
+#ifndef SQ_EPI_HOLD_GR
+#define SQ_EPI_HOLD_GR 2  // 32-column groups a grouped epilogue stores after releasing the accumulator
+#endif
 #ifndef SQ_SCALE_DEPTH
 #define SQ_SCALE_DEPTH 4      // scale bytes are loaded this many of a group's k-steps ahead
 #endif
@@ -1158,70 +1161,129 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           }
           continue;
         }
-        const uint32_t t_buf = t_row + h * kTmemCols;
-        // input gradient and grouped launches: the last 32-column group is read into
-        // registers and stored after the accumulator is released
-        constexpr bool kHold = MODE == MODE_DX || GR;
-        uint32_t held[16];
+        if constexpr (GR) {
+          const uint32_t t_buf = t_row + h * kTmemCols;
+          // the last SQ_EPI_HOLD_GR 32-column groups are read into registers and stored
+          // after the accumulator is released (the loop is unrolled to keep them there)
+          constexpr int kGroups = C::kTile / 2 / 32;
+          constexpr int kHeld = SQ_EPI_HOLD_GR;
+          uint32_t held[kHeld][16];
+          auto store_box = [&](const uint32_t (&w)[16], int c) {
+            if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
+            __syncwarp();
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+            fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
+            __syncwarp();
+            if (lane == 0) {
+              if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
+              bulk_commit_group();
+            }
+          };
+#pragma unroll
+          for (int gi = 0; gi < kGroups; ++gi) {
+            const int c = cbase + 32 * gi;
+            uint32_t v[32];
+            tmem_ld32(t_buf + c, v);
+            tmem_ld_wait();
+            uint32_t packed[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              const __nv_bfloat162 h2 =
+                  __floats2bfloat162_rn(__uint_as_float(v[2 * q]) * scale, __uint_as_float(v[2 * q + 1]) * scale);
+              packed[q] = *reinterpret_cast<const uint32_t *>(&h2);
+            }
+            if (gi >= kGroups - kHeld) {
+#pragma unroll
+              for (int q = 0; q < 16; ++q) held[gi - (kGroups - kHeld)][q] = packed[q];
+            } else {
+              store_box(packed, c);
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          // accumulator h drained: the leader's warps arrive (warp 0 arming the peer's
+          // bytes), the peer's warps signal with a non-blocking async store
+          if (lane == 0) {
+            if (rank == 0) {
+              if (warp == 0)
+                mbar_arrive_expect_tx(&tempty[h], 4 * C::kEpiWarps);
+              else
+                mbar_arrive(&tempty[h]);
+            } else {
+              st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
+                              mapa_shared(smem_u32(&tempty[h]), 0));
+            }
+          }
+#pragma unroll
+          for (int hi = 0; hi < kHeld; ++hi) store_box(held[hi], cbase + 32 * (kGroups - kHeld + hi));
+        } else {
+          const uint32_t t_buf = t_row + h * kTmemCols;
+          // input gradient and grouped launches: the last 32-column group is read into
+          // registers and stored after the accumulator is released
+          constexpr bool kHold = MODE == MODE_DX || GR;
+          uint32_t held[16];
 #pragma unroll 1
-        for (int j = 0; j < C::kTile / 2; j += 32) {
-          const int c = cbase + j;
-          uint32_t v[32];
-          tmem_ld32(t_buf + c, v);
-          tmem_ld_wait();
-          uint32_t packed[16];
+          for (int j = 0; j < C::kTile / 2; j += 32) {
+            const int c = cbase + j;
+            uint32_t v[32];
+            tmem_ld32(t_buf + c, v);
+            tmem_ld_wait();
+            uint32_t packed[16];
 #pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            const __nv_bfloat162 h2 =
-                __floats2bfloat162_rn(__uint_as_float(v[2 * q]) * scale, __uint_as_float(v[2 * q + 1]) * scale);
-            packed[q] = *reinterpret_cast<const uint32_t *>(&h2);
+            for (int q = 0; q < 16; ++q) {
+              const __nv_bfloat162 h2 =
+                  __floats2bfloat162_rn(__uint_as_float(v[2 * q]) * scale, __uint_as_float(v[2 * q + 1]) * scale);
+              packed[q] = *reinterpret_cast<const uint32_t *>(&h2);
+            }
+            if (kHold && j == C::kTile / 2 - 32) {
+#pragma unroll
+              for (int q = 0; q < 16; ++q) held[q] = packed[q];
+              break;
+            }
+            if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
+            __syncwarp();
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), packed[4 * q], packed[4 * q + 1],
+                           packed[4 * q + 2], packed[4 * q + 3]);
+            fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
+            __syncwarp();
+            if (lane == 0) {
+              if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
+              bulk_commit_group();
+            }
           }
-          if (kHold && j == C::kTile / 2 - 32) {
-#pragma unroll
-            for (int q = 0; q < 16; ++q) held[q] = packed[q];
-            break;
-          }
-          if (lane == 0) bulk_wait_read<0>();  // the previous box's store has read the buffer
+          tc_fence_before();
           __syncwarp();
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), packed[4 * q], packed[4 * q + 1],
-                         packed[4 * q + 2], packed[4 * q + 3]);
-          fence_proxy_async_smem();  // the box -> async proxy (the TMA store)
-          __syncwarp();
+          // accumulator h drained: the leader's warps arrive (warp 0 arming the peer's
+          // bytes), the peer's warps signal with a non-blocking async store
           if (lane == 0) {
-            if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
-            bulk_commit_group();
+            if (rank == 0) {
+              if (warp == 0)
+                mbar_arrive_expect_tx(&tempty[h], 4 * C::kEpiWarps);
+              else
+                mbar_arrive(&tempty[h]);
+            } else {
+              st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
+                              mapa_shared(smem_u32(&tempty[h]), 0));
+            }
           }
-        }
-        tc_fence_before();
-        __syncwarp();
-        // accumulator h drained: the leader's warps arrive (warp 0 arming the peer's
-        // bytes), the peer's warps signal with a non-blocking async store
-        if (lane == 0) {
-          if (rank == 0) {
-            if (warp == 0)
-              mbar_arrive_expect_tx(&tempty[h], 4 * C::kEpiWarps);
-            else
-              mbar_arrive(&tempty[h]);
-          } else {
-            st_async_signal(mapa_shared(smem_u32(&sink[2 * C::kDecWarps + warp]), 0),
-                            mapa_shared(smem_u32(&tempty[h]), 0));
-          }
-        }
-        if (kHold) {  // the held group: staged and stored now
-          const int c = cbase + C::kTile / 2 - 32;
-          if (lane == 0) bulk_wait_read<0>();
-          __syncwarp();
+          if (kHold) {  // the held group: staged and stored now
+            const int c = cbase + C::kTile / 2 - 32;
+            if (lane == 0) bulk_wait_read<0>();
+            __syncwarp();
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), held[4 * q], held[4 * q + 1], held[4 * q + 2],
-                         held[4 * q + 3]);
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
-            bulk_commit_group();
+            for (int q = 0; q < 4; ++q)
+              st_shared_v4(row_base + ((q ^ ((lane >> 1) & 3)) << 4), held[4 * q], held[4 * q + 1], held[4 * q + 2],
+                           held[4 * q + 3]);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              if (row < rows && col0 + c < Ng) tma_store_2d(mO, box, col0 + c, row);
+              bulk_commit_group();
+            }
           }
         }
       }
