@@ -1112,9 +1112,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
     // 32 (w % 4) .. +31 and columns 128 (w / 4) .. +127, 32 columns at a time:
     // it scales and rounds them to bf16 into a 32 x 32 box in shared memory
     // (64-byte swizzle) and stores the box with TMA, which writes whole row
-    // segments and clips the ragged edges of the output. The input-gradient and
-    // grouped kernels keep a warp's last group in registers and release the
-    // accumulator before staging it (measured: it helps those, not the forward).
+    // segments and clips the ragged edges of the output. The dense input gradient
+    // keeps a warp's last group in registers and releases the accumulator before
+    // staging it, the grouped kernels their last two groups (measured: it helps
+    // those, not the dense forward; two groups cost the dense input gradient).
     const int quad = warp & 3;
     const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
     const int cbase = (warp >> 2) * (C::kTile / 2);
@@ -1220,9 +1221,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           for (int hi = 0; hi < kHeld; ++hi) store_box(held[hi], cbase + 32 * (kGroups - kHeld + hi));
         } else {
           const uint32_t t_buf = t_row + h * kTmemCols;
-          // input gradient and grouped launches: the last 32-column group is read into
-          // registers and stored after the accumulator is released
-          constexpr bool kHold = MODE == MODE_DX || GR;
+          // the input gradient: the last 32-column group is read into registers and
+          // stored after the accumulator is released
+          constexpr bool kHold = MODE == MODE_DX;
           uint32_t held[16];
 #pragma unroll 1
           for (int j = 0; j < C::kTile / 2; j += 32) {
