@@ -549,10 +549,20 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
     ws2 = __ldg(ws2_per + e);
     cap = 448.0f * ws2;  // the same IEEE fp32 product as the host's single-plane cap
   }
-  for (int i = threadIdx.x; i < kT * r; i += kThreads) {
-    const int row = i / r, j = i % r;
-    const int64_t n = n0 + row;
-    sB[j * kTP + row] = n < N ? bf16_bits(B[n * r + j]) : 0.f;
+  {  // B's rows n0 .. n0 + 63 are kT * r contiguous elements; (row, j) of element i advance
+     // by (kThreads / r, kThreads % r) per step, so no step divides by r
+    int row = static_cast<int>(threadIdx.x) / r, j = static_cast<int>(threadIdx.x) % r;
+    const int drow = kThreads / r, dj = kThreads % r;
+    for (int i = threadIdx.x; i < kT * r; i += kThreads) {
+      const int64_t n = n0 + row;
+      sB[j * kTP + row] = n < N ? bf16_bits(B[n0 * r + i]) : 0.f;
+      row += drow;
+      j += dj;
+      if (j >= r) {
+        j -= r;
+        ++row;
+      }
+    }
   }
   for (int i = threadIdx.x; i < r * kT; i += kThreads) {
     const int64_t b = b0 + i % kT;
@@ -585,18 +595,12 @@ __global__ void __launch_bounds__(kThreads) sq_project_lowrank_kernel(
     const int64_t i0 = n * G + bq;
     if (vec && bq + 3 < G) {
       const uint32_t base4 = __ldg(reinterpret_cast<const uint32_t *>(base + i0));
-      uint32_t by4 = 0, mk4 = 0;
       float Lv[4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const float L = fmaf(aor, acc[q][c], scale_value<FMT>((base4 >> (8 * c)) & 0xFFu, ws2));
-        uint32_t by, mk, na;
-        project_one<FMT>(L, ws2, cap, by, mk, na);
-        by4 |= by << (8 * c);
-        mk4 |= mk << (8 * c);
-        nan_count += na;
-        Lv[c] = L;
-      }
+      for (int c = 0; c < 4; ++c) Lv[c] = fmaf(aor, acc[q][c], scale_value<FMT>((base4 >> (8 * c)) & 0xFFu, ws2));
+      uint32_t by4, mk4, na;
+      project4<FMT>(make_float4(Lv[0], Lv[1], Lv[2], Lv[3]), ws2, cap, by4, mk4, na);
+      nan_count += na;
       *reinterpret_cast<uint32_t *>(bytes_out + i0) = by4;
       if (mask_out) *reinterpret_cast<uint32_t *>(mask_out + i0) = mk4;
       if (latent_out) *reinterpret_cast<float4 *>(latent_out + i0) = make_float4(Lv[0], Lv[1], Lv[2], Lv[3]);
