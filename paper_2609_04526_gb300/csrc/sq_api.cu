@@ -3,6 +3,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -447,6 +448,12 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
   const int64_t N = w->N, K = w->K;
   // the tile list: FWD / DX ceil(M_e / 512) row tiles of each expert x its column
   // tiles; SGRAD every expert's full (N / 256) x (K / 256) grid, empty experts included
+  // table entry x holds expert order[x]: the scale gradient's units of one expert last
+  // M_e tokens, so its entries go longest first; the other modes keep the experts' order
+  std::vector<int> order(E);
+  for (int x = 0; x < E; ++x) order[x] = x;
+  if (mode == sqi::MODE_SGRAD)
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return rows[a] > rows[b]; });
   std::vector<int32_t> tile_start(E + 1, 0);
   int64_t total = 0;
   if (mode == sqi::MODE_SGRAD) {
@@ -460,7 +467,7 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
     const int64_t tn = ((mode == sqi::MODE_FWD ? N : K) + sqi::kPairNTile - 1) / sqi::kPairNTile;
     for (int x = 0; x < E; ++x) {
       tile_start[x] = static_cast<int32_t>(total);
-      total += (rows[x] + sqi::kPairMTile - 1) / sqi::kPairMTile * tn;
+      total += (rows[order[x]] + sqi::kPairMTile - 1) / sqi::kPairMTile * tn;
       if (total > kMaxTokens) return fail(h, SQ_ERR_INVALID_ARG, "too many tiles");
     }
   }
@@ -473,8 +480,9 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
   std::memset(t->host, 0, bytes);
   auto *maps = reinterpret_cast<sqi::GroupMaps *>(t->host);
   for (int x = 0; x < E; ++x) {
-    if (rows[x] == 0) continue;  // no tiles read this expert's descriptors
-    const int64_t m = rows[x], r0 = offsets[x];
+    const int ex = order[x];
+    if (rows[ex] == 0) continue;  // no tiles read this expert's descriptors
+    const int64_t m = rows[ex], r0 = offsets[ex];
     if (mode == sqi::MODE_FWD) {
       SQ_TRY(make_act_map(h, &maps[x].m[0], a_ptr + r0 * K, K, m, 64, sqi::kBM));
       SQ_TRY(make_out_map(h, &maps[x].m[1], static_cast<uint16_t *>(out) + r0 * N, N, m));
@@ -489,10 +497,12 @@ sq_status run_grouped(sq_handle h, int mode, const sq_grouped_weight *w, const s
   auto *ts = reinterpret_cast<int32_t *>(t->host + sqi::group_off_tiles(E));
   auto *rw = reinterpret_cast<int32_t *>(t->host + sqi::group_off_rows(E));
   auto *ws = reinterpret_cast<float *>(t->host + sqi::group_off_ws2(E));
+  auto *id = reinterpret_cast<int32_t *>(t->host + sqi::group_off_ids(E));
   for (int x = 0; x <= E; ++x) ts[x] = tile_start[x];
   for (int x = 0; x < E; ++x) {
-    rw[x] = static_cast<int32_t>(rows[x]);
-    ws[x] = w->ws2 ? w->ws2[x] : 1.0f;
+    rw[x] = static_cast<int32_t>(rows[order[x]]);
+    ws[x] = w->ws2 ? w->ws2[order[x]] : 1.0f;
+    id[x] = order[x];
   }
   // all experts' codes as one [E * N, K/2] tensor, the dense kernels' code boxes
   CUtensorMap tmCodes;

@@ -420,6 +420,9 @@ __device__ __forceinline__ const GroupMaps *group_maps(const KParams &p, int e) 
 __device__ __forceinline__ int group_rows(const KParams &p, int e) {
   return __ldg(reinterpret_cast<const int *>(p.gtab + group_off_rows(p.groups)) + e);
 }
+__device__ __forceinline__ int group_id(const KParams &p, int e) {
+  return __ldg(reinterpret_cast<const int *>(p.gtab + group_off_ids(p.groups)) + e);
+}
 __device__ __forceinline__ float group_ws2(const KParams &p, int e) {
   return __ldg(reinterpret_cast<const float *>(p.gtab + group_off_ws2(p.groups)) + e);
 }
@@ -1492,9 +1495,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(SgradPairCfg::kThrea
       const int num_k = unit_of(tile, e, tm, tn, sp, m0);
       // the expert's code plane (the multiplicative control: its bf16 weights), gradient plane and
       // mask; a token split writes its own partial plane, masked when the parts are added
-      const uint8_t *codes = GR ? p.codes + e * p.N * (p.K / 2) : p.codes;
-      float *g = p.splits > 1 ? p.partial + sp * p.N * G : static_cast<float *>(p.out) + (GR ? e * p.N * G : 0);
-      const uint8_t *mask = p.mask && p.splits == 1 ? p.mask + (GR ? e * p.N * G : 0) : nullptr;
+      const int64_t eid = GR ? group_id(p, e) : 0;  // the expert of table entry e
+      const uint8_t *codes = GR ? p.codes + eid * p.N * (p.K / 2) : p.codes;
+      float *g = p.splits > 1 ? p.partial + sp * p.N * G : static_cast<float *>(p.out) + (GR ? eid * p.N * G : 0);
+      const uint8_t *mask = p.mask && p.splits == 1 ? p.mask + (GR ? eid * p.N * G : 0) : nullptr;
       const bool empty_sum = num_k == 0;  // no tokens: the accumulator was never written
       const int64_t n = static_cast<int64_t>(tm) * C::kTile + 128 * rank + r;
       const int64_t col0 = static_cast<int64_t>(tn) * C::kTile;

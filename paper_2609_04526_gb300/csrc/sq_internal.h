@@ -41,6 +41,10 @@ struct GemmArgs {
 //   int32 tile_start[E+1] first tile of each expert in the launch's tile list
 //   int32 rows[E]        the expert's token count M_e
 //   float ws2[E]         the expert's tensor scale (1.0 for MXFP4)
+//   int32 id[E]          the expert of each entry: the scale gradient lists the experts
+//                        longest first (its units last M_e tokens; dealt round-robin to
+//                        the clusters, equal-length units then share a round), the
+//                        forward and input gradient in order (their tiles are all K long)
 struct GroupMaps {
   CUtensorMap m[2];
 };
@@ -48,7 +52,8 @@ static_assert(sizeof(GroupMaps) == 256, "two 128-byte tensor maps per expert");
 __host__ __device__ constexpr size_t group_off_tiles(int E) { return static_cast<size_t>(E) * sizeof(GroupMaps); }
 __host__ __device__ constexpr size_t group_off_rows(int E) { return group_off_tiles(E) + static_cast<size_t>(E + 1) * 4; }
 __host__ __device__ constexpr size_t group_off_ws2(int E) { return group_off_rows(E) + static_cast<size_t>(E) * 4; }
-__host__ __device__ constexpr size_t group_table_bytes(int E) { return group_off_ws2(E) + static_cast<size_t>(E) * 4; }
+__host__ __device__ constexpr size_t group_off_ids(int E) { return group_off_ws2(E) + static_cast<size_t>(E) * 4; }
+__host__ __device__ constexpr size_t group_table_bytes(int E) { return group_off_ids(E) + static_cast<size_t>(E) * 4; }
 
 // Output rows of one FWD / DX tile and tokens of one scale-gradient stage: the
 // host sizes the grouped tile list with these.
